@@ -1,0 +1,218 @@
+// api.cu -- the extern "C" entry points declared in include/rheo.h.
+//
+// Host side only: argument validation, the workspace layout, kernel selection
+// (dtype x 16-byte alignment) and launches on the caller's stream.  No
+// allocation, no synchronisation except in rheo_get_status.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "rheo.h"
+#include "rheo_device.cuh"
+#include "rheo_kernels.h"
+
+namespace rheo {
+namespace {
+
+int64_t nodes_per_request(const rheo_config& c) {
+    return 1 + (int64_t)(c.K + 1) + (int64_t)(c.depth - 1) * c.K * (c.K + 1);
+}
+int64_t expansions_per_request(const rheo_config& c) { return 1 + (int64_t)(c.depth - 1) * c.K; }
+int elem_size(const rheo_config& c) { return c.dtype == RHEO_BF16 ? 2 : 4; }
+int chunk_elems(const rheo_config& c) { return kChunkBytes / elem_size(c); }
+int chunks_per_row(const rheo_config& c) { return (c.vocab + chunk_elems(c) - 1) / chunk_elems(c); }
+
+bool valid(const rheo_config* c) {
+    if (!c) return false;
+    if (c->dtype != RHEO_F32 && c->dtype != RHEO_BF16) return false;
+    if (c->batch < 1 || c->vocab < 1 || c->vocab > kMaxVocab) return false;
+    if (c->K < 0 || c->m < 0 || c->m > c->K) return false;
+    if (c->support < c->K + 1 || c->support > c->vocab || c->support > kMaxSupport) return false;
+    if (c->depth < 1 || (c->K == 0 && c->depth > 1)) return false;
+    const int64_t G1 = nodes_per_request(*c);
+    if (G1 > kMaxNodes) return false;
+    if (c->budget < 1 || c->budget > G1 - 1) return false;
+    if (c->m == 0 && !(c->eps > 0.0f && c->eps < 1.0f)) return false;
+    const int64_t F = c->K > 0 ? c->K : 1;
+    if ((int64_t)c->batch * F > 65535 || (int64_t)c->batch * (c->budget + 1) > 65535) return false;
+    return true;
+}
+
+struct Layout {
+    size_t status, ex_row_ticket, ex_req_ticket, ex_mu, ex_sum, ex_keys;
+    size_t v_mu, v_sum, v_gather, v_req_ticket, v_desc, v_excl, v_rhat, r_best, r_ticket;
+    size_t total;
+};
+
+size_t up(size_t x) { return (x + 255) & ~(size_t)255; }
+
+Layout layout(const rheo_config& c) {
+    const int64_t B = c.batch, F = c.K > 0 ? c.K : 1, C = chunks_per_row(c), S = c.support;
+    const int64_t NP = c.budget + 1, TL = c.support - c.m, GW = (c.K + 1) + TL;
+    Layout L{};
+    size_t o = 0;
+    auto take = [&](size_t bytes) { size_t at = o; o = up(o + bytes); return at; };
+    L.status = take(sizeof(unsigned));
+    L.ex_row_ticket = take(sizeof(unsigned) * B * F);
+    L.ex_req_ticket = take(sizeof(unsigned) * B);
+    L.ex_mu = take(sizeof(float) * B * F * C);
+    L.ex_sum = take(sizeof(double) * B * F * C);
+    L.ex_keys = take(sizeof(unsigned long long) * B * F * C * S);
+    L.v_mu = take(sizeof(float) * B * NP * C);
+    L.v_sum = take(sizeof(double) * B * NP * C);
+    L.v_gather = take(sizeof(float) * B * NP * GW);
+    L.v_req_ticket = take(sizeof(unsigned) * B);
+    L.v_desc = take(sizeof(int32_t) * B * 8);
+    L.v_excl = take(sizeof(int32_t) * B * (c.K + 1));
+    L.v_rhat = take(sizeof(float) * B * TL);
+    L.r_best = take(sizeof(unsigned long long) * B * 3);
+    L.r_ticket = take(sizeof(unsigned) * B);
+    L.total = o;
+    return L;
+}
+
+Dims dims(const rheo_config& c) {
+    Dims n;
+    n.B = c.batch; n.V = c.vocab; n.K = c.K; n.m = c.m; n.S = c.support; n.D = c.depth; n.N = c.budget;
+    n.TL = c.support - c.m;
+    n.GW = (c.K + 1) + n.TL;
+    n.chunks = chunks_per_row(c);
+    n.G1 = nodes_per_request(c);
+    n.E = expansions_per_request(c);
+    n.eps = c.eps;
+    return n;
+}
+
+bool tree_ok(const rheo_tree* t) {
+    return t && t->token && t->parent && t->log_proxy && t->score && t->qtilde && t->slot && t->frontier &&
+           t->tail_ids && t->tail_q && t->lse1;
+}
+bool pruned_ok(const rheo_pruned* p) {
+    return p && p->gen_id && p->token && p->parent && p->depth && p->first_child && p->n_child && p->sampled_child;
+}
+
+TreePtrs tree_ptrs(const rheo_tree* t) {
+    return TreePtrs{t->token, t->parent, t->log_proxy, t->score, t->qtilde, t->slot,
+                    t->frontier, t->tail_ids, t->tail_q, t->lse1};
+}
+PrunedPtrs pruned_ptrs(const rheo_pruned* p) {
+    return PrunedPtrs{p->gen_id, p->token, p->parent, p->depth, p->first_child, p->n_child, p->sampled_child};
+}
+
+bool aligned16(const void* p, int64_t row_stride, int esize) {
+    return ((uintptr_t)p % 16 == 0) && ((row_stride * esize) % 16 == 0);
+}
+
+template <class T> T* at(void* ws, size_t off) { return reinterpret_cast<T*>(static_cast<char*>(ws) + off); }
+
+}  // namespace
+}  // namespace rheo
+
+using namespace rheo;
+
+extern "C" int rheo_sizes(const rheo_config* cfg, int64_t* nodes, int64_t* expansions, size_t* ws_bytes) {
+    if (!valid(cfg)) return RHEO_EINVAL;
+    if (nodes) *nodes = nodes_per_request(*cfg);
+    if (expansions) *expansions = expansions_per_request(*cfg);
+    if (ws_bytes) *ws_bytes = layout(*cfg).total;
+    return RHEO_OK;
+}
+
+extern "C" int rheo_workspace_init(const rheo_config* cfg, void* ws, size_t bytes, rheo_stream_t stream) {
+    if (!valid(cfg) || !ws || bytes < layout(*cfg).total) return RHEO_EINVAL;
+    return cudaMemsetAsync(ws, 0, layout(*cfg).total, (cudaStream_t)stream) == cudaSuccess ? RHEO_OK : RHEO_ELAUNCH;
+}
+
+extern "C" int rheo_expand(const rheo_config* cfg, int32_t d, const void* logits, int64_t row_stride,
+                           const float* temperature, const uint64_t* seed, const uint64_t* offset,
+                           const rheo_tree* tree, void* ws, rheo_stream_t stream) {
+    if (!valid(cfg) || d < 1 || d > cfg->depth || !logits || row_stride < cfg->vocab || !temperature || !seed ||
+        !offset || !tree_ok(tree) || !ws)
+        return RHEO_EINVAL;
+    const Layout L = layout(*cfg);
+    ExpandArgs a;
+    a.n = dims(*cfg);
+    a.d = d;
+    a.F = (d == 1) ? 1 : cfg->K;
+    a.logits = static_cast<const char*>(logits);
+    a.row_stride_bytes = row_stride * elem_size(*cfg);
+    a.T = temperature;
+    a.seed = seed;
+    a.offset = offset;
+    a.tree = tree_ptrs(tree);
+    a.status = at<unsigned>(ws, L.status);
+    a.row_ticket = at<unsigned>(ws, L.ex_row_ticket);
+    a.req_ticket = at<unsigned>(ws, L.ex_req_ticket);
+    a.chunk_mu = at<float>(ws, L.ex_mu);
+    a.chunk_sum = at<double>(ws, L.ex_sum);
+    a.chunk_keys = at<unsigned long long>(ws, L.ex_keys);
+    const dim3 grid(a.n.chunks, cfg->batch * a.F);
+    const int key_slots = a.n.chunks * cfg->support > kCandCap ? a.n.chunks * cfg->support : kCandCap;
+    const size_t smem = sizeof(unsigned long long) * key_slots;
+    const bool al = aligned16(logits, row_stride, elem_size(*cfg));
+    return launch_expand(a, cfg->dtype, al, grid, smem, (cudaStream_t)stream) == cudaSuccess ? RHEO_OK : RHEO_ELAUNCH;
+}
+
+extern "C" int rheo_prune(const rheo_config* cfg, const rheo_tree* tree, const rheo_pruned* pruned, void* ws,
+                          rheo_stream_t stream) {
+    if (!valid(cfg) || !tree_ok(tree) || !pruned_ok(pruned) || !ws) return RHEO_EINVAL;
+    const Layout L = layout(*cfg);
+    PruneArgs a;
+    a.n = dims(*cfg);
+    a.tree = tree_ptrs(tree);
+    a.pr = pruned_ptrs(pruned);
+    a.status = at<unsigned>(ws, L.status);
+    const size_t smem = sizeof(int32_t) * (size_t)a.n.G1;
+    return launch_prune(a, cfg->batch, smem, (cudaStream_t)stream) == cudaSuccess ? RHEO_OK : RHEO_ELAUNCH;
+}
+
+extern "C" int rheo_verify(const rheo_config* cfg, const void* logits, int64_t row_stride, const float* temperature,
+                           const uint64_t* seed, const uint64_t* offset, const rheo_tree* tree,
+                           const rheo_pruned* pruned, const rheo_verify_out* out, void* ws, rheo_stream_t stream) {
+    if (!valid(cfg) || !logits || row_stride < cfg->vocab || !temperature || !seed || !offset || !tree_ok(tree) ||
+        !pruned_ok(pruned) || !out || !out->accepted_len || !out->accepted_tokens || !out->accepted_nodes ||
+        !out->bonus_token || !ws)
+        return RHEO_EINVAL;
+    const Layout L = layout(*cfg);
+    VerifyArgs a;
+    a.n = dims(*cfg);
+    a.logits = static_cast<const char*>(logits);
+    a.row_stride_bytes = row_stride * elem_size(*cfg);
+    a.T = temperature;
+    a.seed = seed;
+    a.offset = offset;
+    a.tree = tree_ptrs(tree);
+    a.pr = pruned_ptrs(pruned);
+    a.accepted_len = out->accepted_len;
+    a.accepted_tokens = out->accepted_tokens;
+    a.accepted_nodes = out->accepted_nodes;
+    a.bonus_token = out->bonus_token;
+    a.row_lse = out->row_lse;
+    a.status = at<unsigned>(ws, L.status);
+    a.row_mu = at<float>(ws, L.v_mu);
+    a.row_sum = at<double>(ws, L.v_sum);
+    a.gather = at<float>(ws, L.v_gather);
+    a.req_ticket = at<unsigned>(ws, L.v_req_ticket);
+    a.desc = at<int32_t>(ws, L.v_desc);
+    a.excl = at<int32_t>(ws, L.v_excl);
+    a.rhat = at<float>(ws, L.v_rhat);
+    a.res_best = at<unsigned long long>(ws, L.r_best);
+    a.res_ticket = at<unsigned>(ws, L.r_ticket);
+    const dim3 g1(a.n.chunks, cfg->batch * (cfg->budget + 1));
+    const dim3 g2(a.n.chunks, cfg->batch);
+    const bool al = aligned16(logits, row_stride, elem_size(*cfg));
+    return launch_verify(a, cfg->dtype, al, g1, g2, (cudaStream_t)stream) == cudaSuccess ? RHEO_OK : RHEO_ELAUNCH;
+}
+
+extern "C" int rheo_get_status(const rheo_config* cfg, void* ws, rheo_stream_t stream, int32_t* status) {
+    if (!valid(cfg) || !ws || !status) return RHEO_EINVAL;
+    const Layout L = layout(*cfg);
+    cudaStream_t s = (cudaStream_t)stream;
+    unsigned host = 0;
+    if (cudaMemcpyAsync(&host, at<unsigned>(ws, L.status), sizeof(unsigned), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return RHEO_ELAUNCH;
+    if (cudaMemsetAsync(at<unsigned>(ws, L.status), 0, sizeof(unsigned), s) != cudaSuccess) return RHEO_ELAUNCH;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return RHEO_ELAUNCH;
+    *status = (int32_t)host;
+    return RHEO_OK;
+}

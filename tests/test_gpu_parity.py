@@ -1,0 +1,227 @@
+"""GPU parity: the CUDA library against the CPU oracle on the same seeded inputs.
+
+Small cases run the oracle on every request and span several chunks, ragged
+row tails, unaligned rows, massive ties, masked vocabularies and the degenerate
+shapes of the method (K = 0, no pruning, budget 1, m = 0 / 2, tiny support).
+The five benchmark workloads run at full size with the oracle on sampled
+requests (requests are independent, so a sub-batch is an exact check).
+"""
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_21827_gb300 import build, rheo, synth
+import parity_harness as ph
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    build.build()
+    import oracle
+    oracle.build()
+
+
+def _cfg(w: synth.Workload) -> rheo.Config:
+    return rheo.Config(batch=w.batch, vocab=w.vocab, K=w.K, depth=w.depth, budget=w.budget, m=w.m,
+                       support=min(w.support, w.vocab), dtype=w.dtype)
+
+
+def _run(w, draft=None, reqs=None, transform=None, pad=0, max_explained_frac=0.05):
+    draft = draft or synth.make_draft_inputs(w, device="cuda")
+    if transform:
+        transform(draft)
+    cfg = _cfg(w)
+    g = ph.run_gpu(w, draft, cfg, row_stride_pad=pad)
+    assert g.status == 0, f"device status {g.status}"
+    reqs = list(range(w.batch)) if reqs is None else reqs
+    o = ph.run_oracle(w, draft, cfg, reqs)
+    rep = ph.compare(cfg, g, o, reqs)
+    print(w.name, rep)
+    assert rep.ok(), str(rep)
+    assert len(rep.explained) <= max(1, max_explained_frac * len(reqs)), str(rep)
+    return g, o, rep
+
+
+def W(name, **kw):
+    base = dict(name=name, batch=4, vocab=1000, depth=3, K=4, budget=12, dtype="f32", zipf_s=1.1,
+                sigma_draft=0.5, sigma_target=0.5, temperatures=(1.0,), seed=4242)
+    base.update(kw)
+    return synth.Workload(**base)
+
+
+SMALL = [
+    synth.WORKLOADS["tiny"],
+    dataclasses.replace(synth.WORKLOADS["tiny"], name="tiny_b8", batch=8),
+    W("odd_v_bf16", vocab=1001, dtype="bf16", temperatures=(0.7, 1.3)),
+    W("v16_m0", vocab=16, support=16, K=3, m=0, depth=2, budget=6, batch=32),
+    W("v50_m2", vocab=50, support=50, K=5, m=2, depth=3, budget=10, dtype="bf16", batch=16),
+    W("chunks_f32", vocab=40000, K=6, depth=4, budget=20, temperatures=(0.6,)),
+    W("chunks_bf16", vocab=50000, K=6, depth=4, budget=20, dtype="bf16", temperatures=(0.5, 0.8, 1.0)),
+    W("k0", vocab=300, K=0, m=0, depth=1, budget=1, batch=16),
+    W("no_prune", vocab=700, K=3, depth=3, budget=(3 + 1) + 2 * 3 * (3 + 1), batch=6),
+    W("budget1", vocab=700, K=3, depth=3, budget=1, batch=6),
+    W("low_T", vocab=5000, K=5, depth=4, budget=15, temperatures=(0.05,), batch=8),
+    W("m3_small_support", vocab=3000, K=6, m=3, support=12, depth=3, budget=14, batch=8),
+]
+
+
+@pytest.mark.parametrize("w", SMALL, ids=[w.name for w in SMALL])
+def test_parity_small(w):
+    _run(w)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_parity_unaligned_rows(dtype):
+    """rows at a stride of V + 1 elements: scalar loads, same results."""
+    w = W(f"unaligned_{dtype}", vocab=3001, dtype=dtype, batch=4)
+    _run(w, pad=1)
+
+
+def _ties(draft):
+    for r in draft.rows:
+        r.copy_(torch.round(r.float() * 2.0).to(r.dtype))  # half-integer grid: many equal logits
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_parity_massive_ties(dtype):
+    """Equal logits everywhere: the top-S boundary needs the id tie-break and
+    the per-chunk candidate list overflows into the exact register path."""
+    w = W(f"ties_{dtype}", vocab=20000, dtype=dtype, K=5, depth=3, budget=12, batch=4)
+    _run(w, transform=_ties)
+
+
+def _constant(draft):
+    for r in draft.rows:
+        r.zero_()
+
+
+def test_parity_constant_rows():
+    w = W("constant", vocab=9000, dtype="bf16", K=4, depth=2, budget=8, batch=2)
+    _run(w, transform=_constant)
+
+
+def _masked(draft):
+    g = torch.Generator(device="cuda")
+    g.manual_seed(7)
+    for r in draft.rows:
+        mask = torch.rand(r.shape, generator=g, device=r.device) < 0.97
+        mask[..., :8] = False  # keep a few finite logits in every row
+        r.masked_fill_(mask, float("-inf"))
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_parity_masked_vocab(dtype):
+    w = W(f"masked_{dtype}", vocab=4096, dtype=dtype, K=4, depth=3, budget=10, batch=4)
+    _run(w, transform=_masked)
+
+
+def test_replay_is_deterministic_and_offset_moves_draws():
+    w = W("replay", vocab=5000, dtype="bf16", K=5, depth=3, budget=12, batch=8)
+    draft = synth.make_draft_inputs(w, device="cuda")
+    cfg = _cfg(w)
+    a = ph.run_gpu(w, draft, cfg)
+    b = ph.run_gpu(w, draft, cfg)
+    np.testing.assert_array_equal(a.token, b.token)
+    np.testing.assert_array_equal(a.bonus, b.bonus)
+    np.testing.assert_array_equal(a.acc_tok, b.acc_tok)
+    draft.offset += 1
+    c = ph.run_gpu(w, draft, cfg)
+    assert not np.array_equal(a.token, c.token)
+
+
+# --------------------------------------------------------------------------
+# the five workloads at full size, oracle on sampled requests
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("name,reqs", [("llama8b", [0]), ("qwen3_batch", [3, 11]), ("serving_mix", [0, 37]),
+                                       ("stress", [101])])
+def test_parity_full_size_workloads(name, reqs):
+    w = synth.WORKLOADS[name]
+    _run(w, reqs=reqs, max_explained_frac=1.0)
+
+
+# --------------------------------------------------------------------------
+# device status: faults in the data are reported, not trapped
+# --------------------------------------------------------------------------
+
+def _status_of(w, transform, T=None):
+    draft = synth.make_draft_inputs(w, device="cuda")
+    transform(draft)
+    if T is not None:
+        draft.temperature.fill_(T)
+    cfg = _cfg(w)
+    tree, ws = rheo.Tree(cfg), rheo.Workspace(cfg)
+    for d in range(1, cfg.depth + 1):
+        rheo.expand(cfg, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tree, ws)
+    st = rheo.status(cfg, ws)
+    assert rheo.status(cfg, ws) == 0  # cleared by the read
+    return st
+
+
+def test_status_nan_logit():
+    w = W("nan", vocab=2000, batch=2)
+    st = _status_of(w, lambda d: d.rows[0].view(-1)[123].fill_(float("nan")))
+    assert st & rheo.STATUS_BAD_LOGIT
+
+
+def test_status_bad_temperature():
+    w = W("badT", vocab=2000, batch=2)
+    assert _status_of(w, lambda d: None, T=0.0) & rheo.STATUS_BAD_TEMPERATURE
+
+
+def test_status_empty_row():
+    w = W("empty", vocab=2000, batch=2)
+    assert _status_of(w, lambda d: d.rows[0].fill_(float("-inf"))) & rheo.STATUS_EMPTY_ROW
+
+
+def test_invalid_arguments_rejected_before_launch():
+    w = W("args", vocab=2000, batch=2)
+    cfg = _cfg(w)
+    draft = synth.make_draft_inputs(w, device="cuda")
+    tree, ws = rheo.Tree(cfg), rheo.Workspace(cfg)
+    with pytest.raises(rheo.RheoError):
+        rheo.expand(cfg, 0, draft.rows[0], draft.temperature, draft.seed, draft.offset, tree, ws)
+    with pytest.raises(rheo.RheoError):
+        rheo.expand(cfg, 2, draft.rows[0], draft.temperature, draft.seed, draft.offset, tree, ws)
+    bad = dataclasses.replace(cfg, K=200)
+    with pytest.raises(rheo.RheoError):
+        bad.sizes()
+
+
+# --------------------------------------------------------------------------
+# CUDA graph capture of a whole cycle reproduces eager results
+# --------------------------------------------------------------------------
+
+def test_cuda_graph_capture_matches_eager():
+    w = W("graph", vocab=30000, dtype="bf16", K=6, depth=4, budget=20, batch=8)
+    draft = synth.make_draft_inputs(w, device="cuda")
+    cfg = _cfg(w)
+    eager = ph.run_gpu(w, draft, cfg)
+    tgt = None
+    tree, pr, out, ws = rheo.Tree(cfg), rheo.Pruned(cfg), rheo.VerifyOut(cfg), rheo.Workspace(cfg)
+    # targets in the eager tree's pruned order (the captured cycle reproduces that tree)
+    tgt = synth.target_rows(w, draft, [torch.from_numpy(f).cuda() for f in eager.frontiers],
+                            torch.from_numpy(eager.pruned["gen_id"]).cuda())
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(g, stream=s):
+            for d in range(1, cfg.depth + 1):
+                rheo.expand(cfg, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tree, ws, s)
+            rheo.prune(cfg, tree, pr, ws, s)
+            rheo.verify(cfg, tgt, draft.temperature, draft.seed, draft.offset, tree, pr, out, ws, s)
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    assert rheo.status(cfg, ws) == 0
+    np.testing.assert_array_equal(tree.token.cpu().numpy(), eager.token)
+    np.testing.assert_array_equal(pr.gen_id.cpu().numpy(), eager.pruned["gen_id"])
+    np.testing.assert_array_equal(out.accepted_tokens.cpu().numpy(), eager.acc_tok)
+    np.testing.assert_array_equal(out.bonus_token.cpu().numpy(), eager.bonus)

@@ -1,0 +1,427 @@
+"""Benchmark: tree-steps/s of the RheoSampling hot path (expand x D + prune + verify).
+
+One step = D rheo_expand calls, one rheo_prune and one rheo_verify for all B
+requests of the Qwen3-shaped batch workload (B = 16, V = 151,936, bf16, D = 8,
+K = 8 (+1 sampled), N = 48, T = 0.7) on synthetic Zipf(1.2) logits.  Inputs for
+every depth and the target rows are resident in HBM before the timed region
+(515 MB per step, four times the 129 MB L2, so no flush is needed).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--workload NAME]
+
+For N > 1 (torchrun) every rank runs its own replica of the workload on its GPU
+(requests are independent: no data-path collective); the timing is the max
+over ranks and value counts the tree-steps of all ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "tree-steps/sec (expand+prune+verify) at batch B, vocab V; HBM GB/s vs peak"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.path = tempfile.mktemp(prefix="rheo_clocks_", suffix=".csv")
+        self.proc = None
+        self.gpu = gpu_index
+
+    def __enter__(self):
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.fh.close()
+
+    def summary(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        with open(self.path) as f:
+            lines = f.readlines()
+        os.unlink(self.path)
+        return self.parse(lines)
+
+    @staticmethod
+    def parse(lines):
+        """Median SM clock, max clock and active throttle reasons of nvidia-smi CSV lines."""
+        rows = []
+        for line in lines:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for _, _, fl in rows for n, v in zip(names, fl) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+def _dist():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def reduce_max_time(seconds: float, world: int, device=None) -> float:
+    """Max of a per-rank duration over all ranks (no-op for one rank)."""
+    if world == 1:
+        return seconds
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([seconds], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+def oracle_cycle_seconds(w, draft, reqs):
+    """Seconds of one CPU-oracle cycle on requests `reqs` of the workload inputs.
+
+    Expansion and prune are timed, target rows are built (untimed) from the
+    oracle's own pruned tree, then verification is timed."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2609_21827_gb300 import synth
+
+    reqs = list(reqs)
+    ocfg = oracle.Config(B=len(reqs), V=w.vocab, K=w.K, m=w.m, S=min(w.support, w.vocab), D=w.depth, N=w.budget)
+    rows = [r[reqs].float().cpu().numpy() for r in draft.rows]
+    T = draft.temperature.cpu().numpy()[reqs]
+    seed = draft.seed.cpu().numpy().view(np.uint64)[reqs]
+    off = draft.offset.cpu().numpy().view(np.uint64)[reqs]
+    t0 = time.perf_counter()
+    tree = oracle.Tree(ocfg)
+    frontiers = []
+    for d in range(1, w.depth + 1):
+        oracle.expand(ocfg, d, rows[d - 1], T, seed, off, tree)
+        if d < w.depth:
+            frontiers.append(tree.frontier.copy())
+    pr = oracle.prune(ocfg, tree)
+    t_build = time.perf_counter() - t0
+    sub = synth.DraftInputs(w, [r[reqs] for r in draft.rows], draft.temperature[reqs], draft.seed[reqs],
+                            draft.offset[reqs])
+    tgt = synth.target_rows(w, sub, [torch.from_numpy(f) for f in frontiers], torch.from_numpy(pr.gen_id.copy()),
+                            request_ids=reqs).float().cpu().numpy()
+    t1 = time.perf_counter()
+    oracle.verify(ocfg, tgt, T, seed, off, tree, pr)
+    return t_build + (time.perf_counter() - t1)
+
+
+def cpu_baseline(w, draft, budget_s=15.0):
+    """The oracle as it stands, on the host cores, over a bounded sample of requests."""
+    import oracle
+
+    oracle.build()
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    first = oracle_cycle_seconds(w, draft, [0])
+    n = max(1, min(w.batch, int(budget_s / max(first, 1e-3))))
+    secs = oracle_cycle_seconds(w, draft, range(n)) if n > 1 else first
+    per_step = secs * w.batch / n
+    return {"value": 1.0 / per_step, "unit": "tree-steps/s", "cores": min(cores, max(n, w.K)),
+            "kind": "oracle",
+            "sample": f"{n} of {w.batch} requests of one {w.name} cycle ({secs:.1f} s), scaled to the full batch"}
+
+
+def build_inputs(w, device):
+    import torch
+
+    from paper_2609_21827_gb300 import rheo, synth
+
+    draft = synth.make_draft_inputs(w, device=device)
+    cfg = rheo.Config(batch=w.batch, vocab=w.vocab, K=w.K, depth=w.depth, budget=w.budget, m=w.m,
+                      support=min(w.support, w.vocab), dtype=w.dtype)
+    tree, pr, out, ws = rheo.Tree(cfg), rheo.Pruned(cfg), rheo.VerifyOut(cfg, row_lse=False), rheo.Workspace(cfg)
+    frontiers = []
+    for d in range(1, cfg.depth + 1):
+        rheo.expand(cfg, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tree, ws)
+        if d < cfg.depth:
+            frontiers.append(tree.frontier.clone())
+    rheo.prune(cfg, tree, pr, ws)
+    target = synth.target_rows(w, draft, frontiers, pr.gen_id)
+    torch.cuda.synchronize()
+    return cfg, draft, target, tree, pr, out, ws
+
+
+def run_reference(args, w):
+    """--impl reference: the CPU oracle on this machine's host cores, same workload and metric.
+    Each step is a bounded sample (one request of the batch), scaled to B requests."""
+    import torch
+
+    world, rank, local = _dist()
+    if rank != 0:
+        return 0
+    import oracle
+    from paper_2609_21827_gb300 import synth
+
+    oracle.build()
+    device = "cuda" if torch.cuda.is_available() else "cpu"
+    draft = synth.make_draft_inputs(w, device=device)
+    times = []
+    for i in range(args.warmup + args.steps):
+        t = oracle_cycle_seconds(w, draft, [i % w.batch])
+        if i >= args.warmup:
+            times.append(t * w.batch)
+    per_step = sum(times) / len(times)
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    value = 1.0 / per_step
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tree-steps/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_step * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "batch": w.batch, "vocab": w.vocab, "depth": w.depth, "K": w.K,
+                       "budget": w.budget, "logits": w.dtype},
+            "cpu_baseline": {"value": value, "unit": "tree-steps/s", "cores": min(cores, w.K), "kind": "oracle",
+                             "sample": f"1 of {w.batch} requests per step, scaled to the full batch"},
+            "e2e": {"value": value, "unit": "tree-steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--workload", default="qwen3_batch")
+    ap.add_argument("--e2e-steps", type=int, default=50)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    args.warmup = max(3, args.warmup)
+
+    from paper_2609_21827_gb300 import build as lib_build
+    from paper_2609_21827_gb300 import synth
+
+    w = synth.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        return run_reference(args, w)
+
+    import torch
+
+    world, rank, local = _dist()
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    device = f"cuda:{local}" if world > 1 else "cuda:0"
+    torch.cuda.set_device(device)
+    lib_build.build()
+    from paper_2609_21827_gb300 import rheo
+
+    cfg, draft, target, tree, pr, out, ws = build_inputs(w, device)
+    D = cfg.depth
+    esz = 2 if w.dtype == "bf16" else 4
+    exp_rows = [w.batch * (1 if d == 1 else w.K) for d in range(1, D + 1)]
+    expand_bytes = sum(exp_rows) * w.vocab * esz
+    verify_bytes = w.batch * (w.budget + 1) * w.vocab * esz
+
+    stream = torch.cuda.Stream(device=device)
+    stream.wait_stream(torch.cuda.current_stream())
+    try:  # events that become record nodes of the captured graph
+        ev = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(D + 3)]
+        graph_events = True
+    except TypeError:
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(D + 3)]
+        graph_events = False
+
+    def step(s, with_events):
+        if with_events:
+            ev[0].record(s)
+        for d in range(1, D + 1):
+            rheo.expand(cfg, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tree, ws, s)
+            if with_events:
+                ev[d].record(s)
+        rheo.prune(cfg, tree, pr, ws, s)
+        if with_events:
+            ev[D + 1].record(s)
+        rheo.verify(cfg, target, draft.temperature, draft.seed, draft.offset, tree, pr, out, ws, s)
+        if with_events:
+            ev[D + 2].record(s)
+
+    # the whole step as one CUDA graph (11 kernels); per-call events captured as graph nodes
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        step(stream, False)
+        stream.synchronize()
+        with torch.cuda.graph(graph, stream=stream):
+            step(stream, graph_events)
+    for _ in range(args.warmup):
+        graph.replay()
+    torch.cuda.synchronize()
+    assert rheo.status(cfg, ws, stream) == 0
+
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with Clocks(torch.cuda.current_device()) as clk:
+        barrier(world)
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            start.record(stream)
+            for _ in range(args.steps):
+                graph.replay()
+            stop.record(stream)
+        torch.cuda.synchronize()
+        barrier(world)
+    local_s = start.elapsed_time(stop) / 1e3
+    secs = reduce_max_time(local_s, world, device)
+    clocks = clk.summary()
+
+    # per-kernel durations: replays (or eager steps when captured events are not
+    # available) with a synchronise after each, events read every time
+    n_k = min(200, args.steps)
+    exp_ms, prune_ms, ver_ms = 0.0, 0.0, 0.0
+    by_depth = [0.0] * D
+    with torch.cuda.stream(stream):
+        for _ in range(n_k):
+            if graph_events:
+                graph.replay()
+            else:
+                step(stream, True)
+            stream.synchronize()
+            exp_ms += ev[0].elapsed_time(ev[D])
+            for d in range(D):
+                by_depth[d] += ev[d].elapsed_time(ev[d + 1])
+            prune_ms += ev[D].elapsed_time(ev[D + 1])
+            ver_ms += ev[D + 1].elapsed_time(ev[D + 2])
+    exp_ms /= n_k
+    prune_ms /= n_k
+    ver_ms /= n_k
+    assert rheo.status(cfg, ws, stream) == 0
+
+    # end to end through the public API with host buffers: H2D of every input, D2H of the results
+    e2e = None
+    if rank == 0 or world > 1:
+        pin = lambda t: t.cpu().pin_memory()
+        h_rows = [pin(r) for r in draft.rows]
+        h_tgt = pin(target)
+        h_T, h_seed, h_off = pin(draft.temperature), pin(draft.seed), pin(draft.offset)
+        d_rows = [torch.empty_like(r) for r in draft.rows]
+        d_tgt = torch.empty_like(target)
+        d_T, d_seed, d_off = (torch.empty_like(draft.temperature), torch.empty_like(draft.seed),
+                              torch.empty_like(draft.offset))
+        res = [torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
+               for x in (out.accepted_len, out.accepted_tokens, out.bonus_token)]
+        h2d = sum(r.numel() * r.element_size() for r in h_rows) + h_tgt.numel() * h_tgt.element_size() + \
+            sum(x.numel() * x.element_size() for x in (h_T, h_seed, h_off))
+        d2h = sum(x.numel() * x.element_size() for x in res)
+
+        def e2e_step(s):
+            for hr, dr in zip(h_rows, d_rows):
+                dr.copy_(hr, non_blocking=True)
+            d_tgt.copy_(h_tgt, non_blocking=True)
+            d_T.copy_(h_T, non_blocking=True)
+            d_seed.copy_(h_seed, non_blocking=True)
+            d_off.copy_(h_off, non_blocking=True)
+            for d in range(1, D + 1):
+                rheo.expand(cfg, d, d_rows[d - 1], d_T, d_seed, d_off, tree, ws, s)
+            rheo.prune(cfg, tree, pr, ws, s)
+            rheo.verify(cfg, d_tgt, d_T, d_seed, d_off, tree, pr, out, ws, s)
+            for x, h in zip((out.accepted_len, out.accepted_tokens, out.bonus_token), res):
+                h.copy_(x, non_blocking=True)
+
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                e2e_step(stream)
+            stream.synchronize()
+            barrier(world)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(args.e2e_steps):
+                e2e_step(stream)
+            e1.record(stream)
+            stream.synchronize()
+        e2e_s = reduce_max_time(e0.elapsed_time(e1) / 1e3, world, device)
+        e2e = {"value": world * args.e2e_steps / e2e_s, "unit": "tree-steps/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h}
+
+    if rank != 0:
+        return 0
+    peak, peak_kind = _peaks()
+    exp_gbs = expand_bytes / (exp_ms / 1e3) / 1e9
+    ver_gbs = verify_bytes / (ver_ms / 1e3) / 1e9
+    step_gbs = (expand_bytes + verify_bytes) / (secs / args.steps) / 1e9
+    dominant = "expand" if exp_ms >= ver_ms else "verify"
+    ach = exp_gbs if dominant == "expand" else ver_gbs
+    traffic = None
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            traffic = json.load(f).get(f"{w.name}:{dominant}")
+    except Exception:
+        pass
+    cpu = None if args.no_cpu_baseline else cpu_baseline(w, draft)
+    line = {
+        "metric": METRIC, "value": world * args.steps / secs, "unit": "tree-steps/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+        "config": {"workload": w.name, "batch": w.batch, "vocab": w.vocab, "depth": w.depth, "K": w.K,
+                   "budget": w.budget, "temperature": sorted(set(w.temperatures)), "logits": w.dtype,
+                   "bytes_per_step": expand_bytes + verify_bytes, "l2": "inputs 4x larger than L2, no flush",
+                   "parallelism": f"replicas{world}", "cuda_graph": True,
+                   "kernel_timing": "graph event nodes" if graph_events else "eager steps"},
+        "roofline": {"bound": "hbm", "kernel": dominant, "achieved": ach, "peak": peak, "unit": "GB/s",
+                     "frac": ach / peak, "peak_kind": peak_kind, "traffic": traffic},
+        "kernels": {"expand_ms_per_step": exp_ms, "expand_ms_by_depth": [x / n_k for x in by_depth],
+                    "expand_gbs": exp_gbs, "prune_ms": prune_ms,
+                    "verify_ms": ver_ms, "verify_gbs": ver_gbs, "step_gbs": step_gbs,
+                    "step_frac_of_peak": step_gbs / peak},
+        "clocks": clocks,
+        "gpu_launches": args.steps * (D + 3),
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line))
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -5,6 +5,7 @@
 // allocation, no synchronisation except in rheo_get_status.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cstdint>
 
 #include "rheo.h"
@@ -19,8 +20,10 @@ int64_t nodes_per_request(const rheo_config& c) {
 }
 int64_t expansions_per_request(const rheo_config& c) { return 1 + (int64_t)(c.depth - 1) * c.K; }
 int elem_size(const rheo_config& c) { return c.dtype == RHEO_BF16 ? 2 : 4; }
-int chunk_elems(const rheo_config& c) { return kChunkBytes / elem_size(c); }
-int chunks_per_row(const rheo_config& c) { return (c.vocab + chunk_elems(c) - 1) / chunk_elems(c); }
+int tiles_per_row(const rheo_config& c) {
+    const int te = expand_tile_elems(c.dtype == RHEO_BF16 ? 1 : 0);
+    return (c.vocab + te - 1) / te;
+}
 
 bool valid(const rheo_config* c) {
     if (!c) return false;
@@ -40,35 +43,66 @@ bool valid(const rheo_config* c) {
 
 struct Layout {
     size_t status, ex_row_ticket, ex_req_ticket, ex_mu, ex_sum, ex_keys;
-    size_t v_mu, v_sum, v_gather, v_req_ticket, v_desc, v_excl, v_rhat, r_best, r_ticket;
+    size_t v_mu, v_sum, v_row_ticket, v_table, v_rhat, r_best, r_ticket;
     size_t total;
 };
 
 size_t up(size_t x) { return (x + 255) & ~(size_t)255; }
 
 Layout layout(const rheo_config& c) {
-    const int64_t B = c.batch, F = c.K > 0 ? c.K : 1, C = chunks_per_row(c), S = c.support;
-    const int64_t NP = c.budget + 1, TL = c.support - c.m, GW = (c.K + 1) + TL;
+    const int64_t B = c.batch, F = c.K > 0 ? c.K : 1, P = tiles_per_row(c), S = c.support;
+    const int64_t NP = c.budget + 1, TL = c.support - c.m;
     Layout L{};
     size_t o = 0;
     auto take = [&](size_t bytes) { size_t at = o; o = up(o + bytes); return at; };
     L.status = take(sizeof(unsigned));
     L.ex_row_ticket = take(sizeof(unsigned) * B * F);
     L.ex_req_ticket = take(sizeof(unsigned) * B);
-    L.ex_mu = take(sizeof(float) * B * F * C);
-    L.ex_sum = take(sizeof(double) * B * F * C);
-    L.ex_keys = take(sizeof(unsigned long long) * B * F * C * S);
-    L.v_mu = take(sizeof(float) * B * NP * C);
-    L.v_sum = take(sizeof(double) * B * NP * C);
-    L.v_gather = take(sizeof(float) * B * NP * GW);
-    L.v_req_ticket = take(sizeof(unsigned) * B);
-    L.v_desc = take(sizeof(int32_t) * B * 8);
-    L.v_excl = take(sizeof(int32_t) * B * (c.K + 1));
-    L.v_rhat = take(sizeof(float) * B * TL);
+    L.ex_mu = take(sizeof(float) * B * F * P);
+    L.ex_sum = take(2 * sizeof(float) * B * F * P);
+    L.ex_keys = take(sizeof(unsigned long long) * B * F * P * S);
+    L.v_mu = take(sizeof(float) * B * NP * P);
+    L.v_sum = take(2 * sizeof(float) * B * NP * P);
+    L.v_row_ticket = take(sizeof(unsigned) * B * NP);
+    L.v_table = take(sizeof(float) * B * NP * verify_table_width(c.K));
+    L.v_rhat = take(sizeof(float) * B * NP * TL);
     L.r_best = take(sizeof(unsigned long long) * B * 3);
     L.r_ticket = take(sizeof(unsigned) * B);
     L.total = o;
     return L;
+}
+
+int sm_count() {
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
+                                                   cudaSuccess || sms < 1)
+        return 1;
+    return sms;
+}
+
+// persistent grid: two CTAs per SM when the shared memory allows it, never
+// more CTAs than tiles (every CTA then owns at least one tile)
+int persistent_grid(int64_t tiles, size_t dyn_smem) {
+    const int per_sm = (dyn_smem + 16 * 1024) * 2 <= 227 * 1024 ? 2 : 1;
+    const int64_t g = (int64_t)sm_count() * per_sm;
+    return (int)(g < tiles ? g : tiles);
+}
+
+// largest number of segments any row is cut into by the tile split
+int max_segments(int64_t rows, int tpr, int grid) {
+    const int64_t total = rows * tpr;
+    auto owner = [&](int64_t t) { return (int)((t * grid + grid - 1) / total); };
+    int best = 1;
+    for (int64_t r = 0; r < rows; ++r) {
+        const int s = owner(r * tpr + tpr - 1) - owner(r * tpr) + 1;
+        best = s > best ? s : best;
+    }
+    return best;
+}
+
+bool tma_ok(const void* p, int64_t row_stride, const rheo_config& c) {
+    const int es = elem_size(c);
+    return ((uintptr_t)p % 16 == 0) && ((row_stride * es) % 16 == 0) && (((int64_t)c.vocab * es) % 16 == 0);
 }
 
 Dims dims(const rheo_config& c) {
@@ -76,7 +110,7 @@ Dims dims(const rheo_config& c) {
     n.B = c.batch; n.V = c.vocab; n.K = c.K; n.m = c.m; n.S = c.support; n.D = c.depth; n.N = c.budget;
     n.TL = c.support - c.m;
     n.GW = (c.K + 1) + n.TL;
-    n.chunks = chunks_per_row(c);
+    n.chunks = tiles_per_row(c);
     n.G1 = nodes_per_request(c);
     n.E = expansions_per_request(c);
     n.eps = c.eps;
@@ -97,10 +131,6 @@ TreePtrs tree_ptrs(const rheo_tree* t) {
 }
 PrunedPtrs pruned_ptrs(const rheo_pruned* p) {
     return PrunedPtrs{p->gen_id, p->token, p->parent, p->depth, p->first_child, p->n_child, p->sampled_child};
-}
-
-bool aligned16(const void* p, int64_t row_stride, int esize) {
-    return ((uintptr_t)p % 16 == 0) && ((row_stride * esize) % 16 == 0);
 }
 
 template <class T> T* at(void* ws, size_t off) { return reinterpret_cast<T*>(static_cast<char*>(ws) + off); }
@@ -143,14 +173,24 @@ extern "C" int rheo_expand(const rheo_config* cfg, int32_t d, const void* logits
     a.status = at<unsigned>(ws, L.status);
     a.row_ticket = at<unsigned>(ws, L.ex_row_ticket);
     a.req_ticket = at<unsigned>(ws, L.ex_req_ticket);
-    a.chunk_mu = at<float>(ws, L.ex_mu);
-    a.chunk_sum = at<double>(ws, L.ex_sum);
-    a.chunk_keys = at<unsigned long long>(ws, L.ex_keys);
-    const dim3 grid(a.n.chunks, cfg->batch * a.F);
-    const int key_slots = a.n.chunks * cfg->support > kCandCap ? a.n.chunks * cfg->support : kCandCap;
-    const size_t smem = sizeof(unsigned long long) * key_slots;
-    const bool al = aligned16(logits, row_stride, elem_size(*cfg));
-    return launch_expand(a, cfg->dtype, al, grid, smem, (cudaStream_t)stream) == cudaSuccess ? RHEO_OK : RHEO_ELAUNCH;
+    a.seg_mu = at<float>(ws, L.ex_mu);
+    a.seg_sum = at<float>(ws, L.ex_sum);
+    a.seg_keys = at<unsigned long long>(ws, L.ex_keys);
+    const int tpr = tiles_per_row(*cfg);
+    const int64_t rows = (int64_t)cfg->batch * a.F;
+    // two CTAs per SM when the merge buffer of that split still fits, else one
+    int grid = (int)std::min<int64_t>(rows * tpr, 2 * (int64_t)sm_count());
+    int segs = max_segments(rows, tpr, grid);
+    size_t smem = expand_smem_bytes(segs, cfg->support);
+    if ((smem + 16 * 1024) * 2 > 227 * 1024) {
+        grid = (int)std::min<int64_t>(rows * tpr, (int64_t)sm_count());
+        segs = max_segments(rows, tpr, grid);
+        smem = expand_smem_bytes(segs, cfg->support);
+    }
+    return launch_expand(a, cfg->dtype, tma_ok(logits, row_stride, *cfg), grid, smem, (cudaStream_t)stream) ==
+                   cudaSuccess
+               ? RHEO_OK
+               : RHEO_ELAUNCH;
 }
 
 extern "C" int rheo_prune(const rheo_config* cfg, const rheo_tree* tree, const rheo_pruned* pruned, void* ws,
@@ -162,7 +202,8 @@ extern "C" int rheo_prune(const rheo_config* cfg, const rheo_tree* tree, const r
     a.tree = tree_ptrs(tree);
     a.pr = pruned_ptrs(pruned);
     a.status = at<unsigned>(ws, L.status);
-    const size_t smem = sizeof(int32_t) * (size_t)a.n.G1;
+    const size_t smem = (sizeof(int32_t) + sizeof(unsigned long long)) * (size_t)a.n.G1 +
+                        5 * sizeof(int32_t) * (size_t)(cfg->budget + 1);
     return launch_prune(a, cfg->batch, smem, (cudaStream_t)stream) == cudaSuccess ? RHEO_OK : RHEO_ELAUNCH;
 }
 
@@ -189,19 +230,22 @@ extern "C" int rheo_verify(const rheo_config* cfg, const void* logits, int64_t r
     a.bonus_token = out->bonus_token;
     a.row_lse = out->row_lse;
     a.status = at<unsigned>(ws, L.status);
-    a.row_mu = at<float>(ws, L.v_mu);
-    a.row_sum = at<double>(ws, L.v_sum);
-    a.gather = at<float>(ws, L.v_gather);
-    a.req_ticket = at<unsigned>(ws, L.v_req_ticket);
-    a.desc = at<int32_t>(ws, L.v_desc);
-    a.excl = at<int32_t>(ws, L.v_excl);
-    a.rhat = at<float>(ws, L.v_rhat);
+    a.seg_mu = at<float>(ws, L.v_mu);
+    a.seg_sum = at<float>(ws, L.v_sum);
+    a.row_ticket = at<unsigned>(ws, L.v_row_ticket);
+    a.table = at<float>(ws, L.v_table);
+    a.rhat_tail = at<float>(ws, L.v_rhat);
     a.res_best = at<unsigned long long>(ws, L.r_best);
     a.res_ticket = at<unsigned>(ws, L.r_ticket);
-    const dim3 g1(a.n.chunks, cfg->batch * (cfg->budget + 1));
-    const dim3 g2(a.n.chunks, cfg->batch);
-    const bool al = aligned16(logits, row_stride, elem_size(*cfg));
-    return launch_verify(a, cfg->dtype, al, g1, g2, (cudaStream_t)stream) == cudaSuccess ? RHEO_OK : RHEO_ELAUNCH;
+    const int64_t NP = cfg->budget + 1;
+    const size_t stage = (size_t)NP * (verify_table_width(cfg->K) * 4 + 5 * 4);
+    a.table_smem_bytes = stage <= 160 * 1024 ? stage : 0;
+    const int tpr = tiles_per_row(*cfg);
+    const int grid = persistent_grid((int64_t)cfg->batch * NP * tpr, verify_stream_smem_bytes());
+    return launch_verify(a, cfg->dtype, tma_ok(logits, row_stride, *cfg), grid, verify_stream_smem_bytes(),
+                         (cudaStream_t)stream) == cudaSuccess
+               ? RHEO_OK
+               : RHEO_ELAUNCH;
 }
 
 extern "C" int rheo_get_status(const rheo_config* cfg, void* ws, rheo_stream_t stream, int32_t* status) {

@@ -1,107 +1,95 @@
 // prune.cu -- global rerank/prune to the verification budget (App. C.1 "Path
 // scores and global pruning"; Lemma 2 makes the result ancestor-closed).
 //
-// One CTA per request.  Keys (ord(score) << 32 | ~gen) order nodes by score
-// descending, then gen id ascending (= shallower first, then left to right);
-// the N-th largest key is found by bitwise selection, the survivors are
-// compacted in gen-id order with a block scan, and parents are remapped
-// through a gen -> pruned-index table in shared memory.
+// One CTA per request, everything staged in shared memory.  Keys
+// (ord(score) << 32 | ~gen) order nodes by score descending, then gen id
+// ascending (= shallower first, then left to right); the N-th largest key is
+// found by bitwise selection, the survivors are compacted in gen-id order with
+// a block scan, and parents are remapped through a gen -> pruned-index table.
 #include "rheo_device.cuh"
 #include "rheo_kernels.h"
 
 namespace rheo {
 
 __global__ void __launch_bounds__(kThreads) prune_kernel(const PruneArgs a) {
-    extern __shared__ int32_t map[];  // [G1]
+    extern __shared__ __align__(16) unsigned char psm[];
     __shared__ BlockScratch bs;
+    __shared__ unsigned hist[kRadixBins];
+    __shared__ RadixScratch rad;
     const Dims& n = a.n;
     const int tid = threadIdx.x;
     const int b = blockIdx.x;
-    const int N = n.N;
-    const int64_t G1 = n.G1;
-    const int64_t nb = (int64_t)b * G1, pb = (int64_t)b * (N + 1);
-    int parity = 0;
+    const int N = n.N, NP = n.N + 1;
+    const int G1 = (int)n.G1;
+    const int64_t nb = (int64_t)b * G1, pb = (int64_t)b * NP;
 
-    auto key_of = [&](int64_t g) -> unsigned long long {
-        return ((unsigned long long)ord_f32(a.tree.score[nb + g]) << 32) | (0xFFFFFFFFu - (uint32_t)g);
-    };
+    unsigned long long* keys = reinterpret_cast<unsigned long long*>(psm);     // [G1]
+    int32_t* map = reinterpret_cast<int32_t*>(keys + G1);                      // [G1] gen -> pruned index
+    int32_t* pgen = map + G1;                                                  // [NP] pruned index -> gen
+    int32_t* ppar = pgen + NP;                                                 // [NP] parent (pruned index)
+    int32_t* pfc = ppar + NP;                                                  // [NP] first child
+    int32_t* plc = pfc + NP;                                                   // [NP] last child
+    int32_t* psc = plc + NP;                                                   // [NP] sampled child
+
+    for (int g = tid; g < G1; g += kThreads)
+        keys[g] = ((unsigned long long)ord_f32(a.tree.score[nb + g]) << 32) | (0xFFFFFFFFu - (uint32_t)g);
+    for (int i = tid; i < NP; i += kThreads) { pfc[i] = -1; plc[i] = -1; psc[i] = -1; }
+    __syncthreads();
 
     // threshold: the N-th largest key among gen ids 1..G1-1
     unsigned long long thr = 1ull;
-    if (G1 - 1 > N) {
-        unsigned long long aand = ~0ull, aor = 0ull;
-        for (int64_t g = 1 + tid; g < G1; g += kThreads) {
-            const unsigned long long x = key_of(g);
-            aand &= x;
-            aor |= x;
-        }
-        aand = block_and_or_u64(aand, false, bs);
-        aor = block_and_or_u64(aor, true, bs);
-        thr = block_select(
-            [&](unsigned long long t) {
-                int c = 0;
-                for (int64_t g = 1 + tid; g < G1; g += kThreads) c += key_of(g) >= t;
-                return c;
-            },
-            N, aand, aor, bs, parity);
-    }
+    if (G1 - 1 > N) thr = block_radix_threshold([&](int i) { return keys[1 + i]; }, G1 - 1, N, hist, rad);
 
     // compaction in gen-id order; the root is always kept
-    const int per = (int)((G1 + kThreads - 1) / kThreads);
-    const int64_t lo = min(G1, (int64_t)tid * per), hi = min(G1, lo + per);
+    const int per = (G1 + kThreads - 1) / kThreads;
+    const int lo = min(G1, tid * per), hi = min(G1, lo + per);
     int cnt = 0;
-    for (int64_t g = lo; g < hi; ++g) cnt += (g == 0 || key_of(g) >= thr);
+    for (int g = lo; g < hi; ++g) cnt += (g == 0 || keys[g] >= thr);
     int total;
     int pos = block_exclusive_scan(cnt, total, bs);
-    for (int64_t g = lo; g < hi; ++g) {
-        if (g == 0 || key_of(g) >= thr) {
+    if (total != NP) {  // cannot happen with distinct keys; never index with a partial table
+        if (tid == 0) atomicOr(a.status, kStInternal);
+        return;
+    }
+    for (int g = lo; g < hi; ++g) {
+        if (g == 0 || keys[g] >= thr) {
             map[g] = pos;
-            if (pos <= N) {
-                a.pr.gen_id[pb + pos] = (int32_t)g;
-                a.pr.token[pb + pos] = a.tree.token[nb + g];
-                a.pr.depth[pb + pos] = depth_of(n.K, g);
-            }
+            pgen[pos] = g;
             ++pos;
         } else {
             map[g] = -1;
         }
     }
-    if (total != N + 1) {  // cannot happen with distinct keys; never index with a partial table
-        if (tid == 0) atomicOr(a.status, kStInternal);
-        return;
-    }
-    for (int i = tid; i <= N; i += kThreads) {
-        a.pr.first_child[pb + i] = -1;
-        a.pr.n_child[pb + i] = 0;
-        a.pr.sampled_child[pb + i] = -1;
-    }
     __syncthreads();
 
-    // parents; children are contiguous in pruned order (gen-consecutive pools)
-    for (int i = tid; i <= N; i += kThreads) {
-        const int64_t g = a.pr.gen_id[pb + i];
+    // parents (one parallel round trip for the tree fields), then children ranges
+    for (int i = tid; i < NP; i += kThreads) {
+        const int g = pgen[i];
         int32_t p = -1;
         if (g != 0) {
             const int32_t pg = a.tree.parent[nb + g];
             p = (pg >= 0 && pg < G1) ? map[pg] : -1;
             if (p < 0) atomicOr(a.status, kStInternal);  // not ancestor-closed (or tree never expanded)
         }
+        ppar[i] = p;
+        a.pr.gen_id[pb + i] = g;
+        a.pr.token[pb + i] = a.tree.token[nb + g];
+        a.pr.depth[pb + i] = depth_of(n.K, g);
         a.pr.parent[pb + i] = p;
     }
     __syncthreads();
-    for (int i = 1 + tid; i <= N; i += kThreads) {
-        const int32_t p = a.pr.parent[pb + i];
+    for (int i = 1 + tid; i < NP; i += kThreads) {
+        const int32_t p = ppar[i];
         if (p < 0) continue;
-        const bool first = (i == 1) || (a.pr.parent[pb + i - 1] != p);
-        const bool last = (i == N) || (a.pr.parent[pb + i + 1] != p);
-        if (first) a.pr.first_child[pb + p] = i;
-        if (last) a.pr.n_child[pb + p] = i;  // index of the last child, turned into a count below
-        if (a.tree.slot[nb + a.pr.gen_id[pb + i]] == kSlotSampled) a.pr.sampled_child[pb + p] = i;
+        if (i == 1 || ppar[i - 1] != p) pfc[p] = i;
+        if (i == N || ppar[i + 1] != p) plc[p] = i;
+        if (a.tree.slot[nb + pgen[i]] == kSlotSampled) psc[p] = i;
     }
     __syncthreads();
-    for (int i = tid; i <= N; i += kThreads) {
-        const int fc = a.pr.first_child[pb + i];
-        if (fc >= 0) a.pr.n_child[pb + i] = a.pr.n_child[pb + i] - fc + 1;
+    for (int i = tid; i < NP; i += kThreads) {
+        a.pr.first_child[pb + i] = pfc[i];
+        a.pr.n_child[pb + i] = (pfc[i] >= 0) ? plc[i] - pfc[i] + 1 : 0;
+        a.pr.sampled_child[pb + i] = psc[i];
     }
 }
 

@@ -53,6 +53,12 @@ template <> struct Elem<0> {
         return __uint_as_float(r);
     }
     __device__ static __forceinline__ uint32_t neg_inf_raw() { return 0xFF800000u; }
+    // key of a value read from this element type
+    __device__ static __forceinline__ uint32_t key_of_value(float x) { return key(__float_as_uint(x)); }
+    // value with the same order as a threshold key; keys at or below key(-inf) give -inf
+    __device__ static __forceinline__ float threshold_value(uint32_t k) {
+        return k <= 0x007FFFFFu ? -INFINITY : value_of_key(k);
+    }
     __device__ static __forceinline__ uint32_t load_scalar(const char* row, int64_t e) {
         return __ldg(reinterpret_cast<const uint32_t*>(row) + e);
     }
@@ -78,6 +84,10 @@ template <> struct Elem<1> {
         return __uint_as_float(h << 16);
     }
     __device__ static __forceinline__ uint32_t neg_inf_raw() { return 0xFF80u; }
+    __device__ static __forceinline__ uint32_t key_of_value(float x) { return key(__float_as_uint(x) >> 16); }
+    __device__ static __forceinline__ float threshold_value(uint32_t k) {
+        return k <= 0x007F0000u ? -INFINITY : value_of_key(k);
+    }
     __device__ static __forceinline__ uint32_t load_scalar(const char* row, int64_t e) {
         return (uint32_t)__ldg(reinterpret_cast<const unsigned short*>(row) + e);
     }
@@ -117,6 +127,57 @@ __device__ __forceinline__ float fast_exp2(float x) {
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
 }
+
+// ---------------------------------------------------------------------------
+// 16-byte vectors of logits: max, partition-sum terms, tail masking
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
+    uint32_t r;
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+    return r;
+}
+__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+template <int DT> struct Vec;
+template <> struct Vec<1> {
+    __device__ static __forceinline__ float vmax(const uint4& v) {
+        const uint32_t m = bmax2(bmax2(v.x, v.y), bmax2(v.z, v.w));
+        return fmaxf(bf_lo(m), bf_hi(m));
+    }
+    // sum of 2^(x c - mc) over the 8 values (independent partial sums)
+    __device__ static __forceinline__ float vexp(const uint4& v, float c, float mc) {
+        const float a0 = fast_exp2(fmaf(bf_lo(v.x), c, -mc)) + fast_exp2(fmaf(bf_hi(v.x), c, -mc));
+        const float a1 = fast_exp2(fmaf(bf_lo(v.y), c, -mc)) + fast_exp2(fmaf(bf_hi(v.y), c, -mc));
+        const float a2 = fast_exp2(fmaf(bf_lo(v.z), c, -mc)) + fast_exp2(fmaf(bf_hi(v.z), c, -mc));
+        const float a3 = fast_exp2(fmaf(bf_lo(v.w), c, -mc)) + fast_exp2(fmaf(bf_hi(v.w), c, -mc));
+        return (a0 + a1) + (a2 + a3);
+    }
+    // elements [nv, 8) become -inf
+    __device__ static __forceinline__ uint4 mask(uint4 v, int nv) {
+        auto m = [](uint32_t w, int lo_idx, int nv) -> uint32_t {
+            if (lo_idx >= nv) return 0xFF80FF80u;
+            if (lo_idx + 1 >= nv) return (w & 0xFFFFu) | 0xFF800000u;
+            return w;
+        };
+        return make_uint4(m(v.x, 0, nv), m(v.y, 2, nv), m(v.z, 4, nv), m(v.w, 6, nv));
+    }
+};
+template <> struct Vec<0> {
+    __device__ static __forceinline__ float vmax(const uint4& v) {
+        return fmaxf(fmaxf(__uint_as_float(v.x), __uint_as_float(v.y)),
+                     fmaxf(__uint_as_float(v.z), __uint_as_float(v.w)));
+    }
+    __device__ static __forceinline__ float vexp(const uint4& v, float c, float mc) {
+        const float a0 = fast_exp2(fmaf(__uint_as_float(v.x), c, -mc)) + fast_exp2(fmaf(__uint_as_float(v.y), c, -mc));
+        const float a1 = fast_exp2(fmaf(__uint_as_float(v.z), c, -mc)) + fast_exp2(fmaf(__uint_as_float(v.w), c, -mc));
+        return a0 + a1;
+    }
+    __device__ static __forceinline__ uint4 mask(uint4 v, int nv) {
+        const uint32_t ni = 0xFF800000u;
+        return make_uint4(nv > 0 ? v.x : ni, nv > 1 ? v.y : ni, nv > 2 ? v.z : ni, nv > 3 ? v.w : ni);
+    }
+};
 
 __device__ __forceinline__ uint32_t ord_f32(float x) { return Elem<0>::key(__float_as_uint(x)); }
 
@@ -162,8 +223,8 @@ __device__ __forceinline__ float gumbel(float u) { return -logf(-logf(u)); }
 // ---------------------------------------------------------------------------
 struct BlockScratch {
     int ired[2][kWarps];
-    double dred[kWarps];
     float fred[kWarps];
+    float fred2[kWarps];
     unsigned long long ured[kWarps];
     int flag;
 };
@@ -220,54 +281,185 @@ __device__ __forceinline__ unsigned long long block_and_or_u64(unsigned long lon
     return t;
 }
 
-// (max, sum of exp relative to max): merged in fp64
-__device__ __forceinline__ void block_max_sum(float mu, double sum, BlockScratch& s, float& out_mu,
-                                              double& out_sum) {
-    float m = mu;
+// block-wide maximum (all threads get it)
+__device__ __forceinline__ float block_max_f32(float v, BlockScratch& s) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
     __syncthreads();
-    if ((threadIdx.x & 31) == 0) s.fred[threadIdx.x >> 5] = m;
+    if ((threadIdx.x & 31) == 0) s.fred[threadIdx.x >> 5] = v;
     __syncthreads();
-    float M = s.fred[0];
+    float m = s.fred[0];
 #pragma unroll
-    for (int w = 1; w < kWarps; ++w) M = fmaxf(M, s.fred[w]);
-    double t = (sum > 0.0) ? sum * exp((double)mu - (double)M) : 0.0;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xFFFFFFFFu, t, o);
-    if ((threadIdx.x & 31) == 0) s.dred[threadIdx.x >> 5] = t;
-    __syncthreads();
-    double T = 0.0;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) T += s.dred[w];
-    out_mu = M;
-    out_sum = T;
+    for (int w = 1; w < kWarps; ++w) m = fmaxf(m, s.fred[w]);
+    return m;
 }
 
 // ---------------------------------------------------------------------------
-// Selection: the k-th largest of a set of 64-bit keys spread over the block.
-// count_ge(t) returns how many of the calling thread's keys are >= t.  and_all
-// / or_all are the bitwise AND / OR of every key.  Returns a threshold T with
-// count(keys >= T) == k when keys are distinct (and the k-th largest value when
-// they are not).  Bits that are equal in every key are copied without a step.
+// float-float arithmetic (value = hi + lo, ~48 significant bits) in place of
+// fp64, whose throughput on this part is a tiny fraction of fp32's.  The
+// explicit _rn intrinsics keep the compiler from contracting the error terms.
 // ---------------------------------------------------------------------------
-template <class CountGE>
-__device__ unsigned long long block_select(CountGE count_ge, int k, unsigned long long and_all,
-                                           unsigned long long or_all, BlockScratch& s, int& parity) {
-    unsigned long long prefix = 0;
-    const unsigned long long fixed = ~(and_all ^ or_all);
-    for (int bit = 63; bit >= 0; --bit) {
-        const unsigned long long mask = 1ull << bit;
-        if (fixed & mask) {
-            prefix |= (and_all & mask);
-            continue;
+struct FF {
+    float hi, lo;
+};
+__device__ __forceinline__ FF ff_two_sum(float a, float b) {
+    const float s = __fadd_rn(a, b);
+    const float bb = __fsub_rn(s, a);
+    const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+    return {s, e};
+}
+__device__ __forceinline__ FF ff_norm(float a, float b) {  // |a| >= |b|
+    const float s = __fadd_rn(a, b);
+    return {s, __fsub_rn(b, __fsub_rn(s, a))};
+}
+__device__ __forceinline__ FF ff_add(FF x, FF y) {
+    if (!(x.hi > -INFINITY && x.hi < INFINITY) || !(y.hi > -INFINITY && y.hi < INFINITY))
+        return {__fadd_rn(x.hi, y.hi), 0.0f};
+    const FF s = ff_two_sum(x.hi, y.hi);
+    return ff_norm(s.hi, __fadd_rn(s.lo, __fadd_rn(x.lo, y.lo)));
+}
+__device__ __forceinline__ FF ff_add(FF x, float y) { return ff_add(x, FF{y, 0.0f}); }
+__device__ __forceinline__ FF ff_neg(FF x) { return {-x.hi, -x.lo}; }
+__device__ __forceinline__ FF ff_shfl_xor(FF x, int o) {
+    return {__shfl_xor_sync(0xFFFFFFFFu, x.hi, o), __shfl_xor_sync(0xFFFFFFFFu, x.lo, o)};
+}
+// a * x exactly enough: (p + e) with e the fma residue
+__device__ __forceinline__ FF ff_mul(float a, FF x) {
+    const float p = __fmul_rn(a, x.hi);
+    const float e = fmaf(a, x.hi, -p);
+    return ff_norm(p, fmaf(a, x.lo, e));
+}
+// log of a positive float-float (first-order correction of logf)
+__device__ __forceinline__ FF ff_log(FF x) {
+    const float y = logf(x.hi);
+    if (!(x.hi > 0.0f) || !(y > -INFINITY && y < INFINITY)) return {y, 0.0f};
+    return ff_two_sum(y, __fdiv_rn(x.lo, x.hi));
+}
+// v / T as float-float: correctly rounded quotient plus the exact fma remainder
+__device__ __forceinline__ FF ff_div(float v, float T) {
+    const float q = __fdiv_rn(v, T);
+    if (!(q > -INFINITY && q < INFINITY)) return {q, 0.0f};
+    return {q, __fdiv_rn(fmaf(-q, T, v), T)};
+}
+// "a <= b" for b a float and a = x (float-float), decided exactly enough
+__device__ __forceinline__ bool ff_le(FF x, float b) {
+    const float d = __fsub_rn(b, x.hi);
+    return d > x.lo || (d == x.lo);
+}
+
+// block-wide sum of fp32 values: float-float (compensated) in and across warps
+__device__ __forceinline__ FF block_sum_ff(FF v, BlockScratch& s) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = ff_add(v, ff_shfl_xor(v, o));
+    __syncthreads();
+    if ((threadIdx.x & 31) == 0) {
+        s.fred[threadIdx.x >> 5] = v.hi;
+        s.fred2[threadIdx.x >> 5] = v.lo;
+    }
+    __syncthreads();
+    FF t{s.fred[0], s.fred2[0]};
+#pragma unroll
+    for (int w = 1; w < kWarps; ++w) t = ff_add(t, FF{s.fred[w], s.fred2[w]});
+    return t;
+}
+__device__ __forceinline__ FF block_sum_ff(float v, BlockScratch& s) { return block_sum_ff(FF{v, 0.0f}, s); }
+
+// exp(l / T - c) for an fp32 logit l and a float-float constant c, to a few
+// fp32 ulps: l / T = tau + rem / T exactly (tau correctly rounded).
+__device__ __forceinline__ float exp_scaled_minus(float l, float T, FF c) {
+    const FF x = ff_div(l, T);
+    if (!(x.hi > -INFINITY && x.hi < INFINITY)) return expf(x.hi - c.hi);
+    const float d = __fsub_rn(x.hi, c.hi) + (x.lo - c.lo);
+    return expf(d);
+}
+
+// ---------------------------------------------------------------------------
+// Selection: threshold T with count(keys >= T) == k for k <= n distinct 64-bit
+// keys spread over the block (for keys with repeats: the k-th largest key).
+// Bits shared by every key are taken from their AND at once; the rest is a
+// radix select on 8-bit digits, most significant first: a shared histogram per
+// digit, a block scan over the digits from the top, stop as soon as the keys
+// at or above the current prefix number exactly k.  get(i), i in [0, n)
+// visited as i = tid + j * kThreads, returns a key, or 0 for "no key".
+// ---------------------------------------------------------------------------
+constexpr int kRadixBins = 256;
+static_assert(kRadixBins == kThreads, "one radix bin per thread");
+
+struct RadixScratch {
+    unsigned long long red_and[kWarps], red_or[kWarps];
+    int wsum[kWarps];
+    int digit, above;
+};
+
+template <class Get>
+__device__ unsigned long long block_radix_threshold(Get get, int n, int k, unsigned* hist, RadixScratch& rs) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    // common leading bits
+    unsigned long long a_and = ~0ull, a_or = 0ull;
+    for (int i = tid; i < n; i += kThreads) {
+        const unsigned long long x = get(i);
+        if (x) { a_and &= x; a_or |= x; }
+    }
+    {
+        unsigned lo_a = __reduce_and_sync(0xFFFFFFFFu, (unsigned)a_and), hi_a = __reduce_and_sync(0xFFFFFFFFu, (unsigned)(a_and >> 32));
+        unsigned lo_o = __reduce_or_sync(0xFFFFFFFFu, (unsigned)a_or), hi_o = __reduce_or_sync(0xFFFFFFFFu, (unsigned)(a_or >> 32));
+        if (lane == 0) {
+            rs.red_and[warp] = ((unsigned long long)hi_a << 32) | lo_a;
+            rs.red_or[warp] = ((unsigned long long)hi_o << 32) | lo_o;
         }
-        const unsigned long long t = prefix | mask;
-        const int c = block_sum_int(count_ge(t), s, parity);
-        if (c >= k) {
-            prefix = t;
-            if (c == k) return prefix;
+        __syncthreads();
+        a_and = ~0ull;
+        a_or = 0ull;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) { a_and &= rs.red_and[w]; a_or |= rs.red_or[w]; }
+    }
+    const unsigned long long diff = a_and ^ a_or;
+    if (diff == 0ull) {  // all keys equal
+        __syncthreads();
+        return a_and;
+    }
+    int top = 64 - __clzll((long long)diff);  // bits >= top are common to every key
+    unsigned long long prefix = (top >= 64) ? 0ull : (a_and >> top) << top;
+    int above = 0;
+    while (top > 0) {
+        const int bits = top >= 8 ? 8 : top;
+        const int shift = top - bits;
+        const unsigned mask = (1u << bits) - 1u;
+        hist[tid] = 0u;  // kThreads == kRadixBins
+        __syncthreads();
+        for (int i = tid; i < n; i += kThreads) {
+            const unsigned long long x = get(i);
+            if (x == 0ull) continue;
+            if (top < 64 && (x >> top) != (prefix >> top)) continue;
+            atomicAdd(&hist[(unsigned)(x >> shift) & mask], 1u);
         }
+        __syncthreads();
+        // thread t owns digit 255 - t (descending order of digits)
+        const int d = kRadixBins - 1 - tid;
+        const int h = (int)hist[d];
+        int incl = h;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        if (lane == 31) rs.wsum[warp] = incl;
+        __syncthreads();
+        int before = above + incl - h;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) before += (w < warp) ? rs.wsum[w] : 0;
+        if (before < k && before + h >= k) {
+            rs.digit = d;
+            rs.above = before;
+        }
+        __syncthreads();
+        const int dd = rs.digit;
+        above = rs.above;
+        prefix |= (unsigned long long)dd << shift;
+        const bool exact = above + (int)hist[dd] == k;
+        __syncthreads();  // everybody has read rs and hist before they change
+        top = shift;
+        if (exact) break;
     }
     return prefix;
 }
@@ -311,23 +503,18 @@ __device__ __forceinline__ bool arrive_last(unsigned* counter, unsigned total, B
     return last;
 }
 
-// numbering helpers (see rheo.h)
-__device__ __forceinline__ int64_t depth_base(int K, int d) {
-    return d == 1 ? 1 : 1 + (int64_t)(K + 1) + (int64_t)(d - 2) * K * (K + 1);
-}
-__device__ __forceinline__ int slot_of(int K, int64_t g) {
-    if (g <= K + 1) return (int)(g - 1);
-    return (int)((g - (K + 2)) % (K + 1));
-}
-__device__ __forceinline__ int64_t parent_expansion_of(int K, int64_t g) {
+// numbering helpers (see rheo.h); gen ids < 2^14, so 32-bit arithmetic
+__device__ __forceinline__ int depth_base(int K, int d) { return d == 1 ? 1 : 1 + (K + 1) + (d - 2) * K * (K + 1); }
+__device__ __forceinline__ int slot_of(int K, int g) { return g <= K + 1 ? g - 1 : (g - (K + 2)) % (K + 1); }
+__device__ __forceinline__ int parent_expansion_of(int K, int g) {
     if (g <= K + 1) return 0;
-    const int64_t w = g - (K + 2), per = (int64_t)K * (K + 1);
+    const int w = g - (K + 2), per = K * (K + 1);
     return 1 + (w / per) * K + (w % per) / (K + 1);
 }
-__device__ __forceinline__ int depth_of(int K, int64_t g) {
+__device__ __forceinline__ int depth_of(int K, int g) {
     if (g == 0) return 0;
     if (g <= K + 1) return 1;
-    return 2 + (int)((g - (K + 2)) / ((int64_t)K * (K + 1)));
+    return 2 + (g - (K + 2)) / (K * (K + 1));
 }
 
 }  // namespace rheo

@@ -48,11 +48,11 @@ struct ExpandArgs {
     const uint64_t* offset;
     TreePtrs tree;
     unsigned* status;
-    unsigned* row_ticket;          // [B*F]
-    unsigned* req_ticket;          // [B]
-    float* chunk_mu;               // [B*F*chunks]
-    double* chunk_sum;             // [B*F*chunks]
-    unsigned long long* chunk_keys;  // [B*F*chunks*S]
+    unsigned* row_ticket;           // [B*F]
+    unsigned* req_ticket;           // [B]
+    float* seg_mu;                  // [B*F*tiles_per_row]
+    float* seg_sum;                 // [B*F*tiles_per_row*2] float-float partition sums
+    unsigned long long* seg_keys;   // [B*F*tiles_per_row*S]
 };
 
 struct PruneArgs {
@@ -75,24 +75,28 @@ struct VerifyArgs {
     int32_t* accepted_tokens;
     int32_t* accepted_nodes;
     int32_t* bonus_token;
-    float* row_lse;  // may be null
+    float* row_lse;                 // may be null
     unsigned* status;
-    float* row_mu;           // [B*(N+1)*chunks]
-    double* row_sum;         // [B*(N+1)*chunks]
-    float* gather;           // [B*(N+1)*GW]
-    unsigned* req_ticket;    // [B]
-    int32_t* desc;           // [B*8]: stop row, gen, lse bits, use_tail, n_excl, expansion, M bits, -
-    int32_t* excl;           // [B*(K+1)]
-    float* rhat;             // [B*TL]
-    unsigned long long* res_best;  // [B*3]
-    unsigned* res_ticket;    // [B]
+    float* seg_mu;                  // [B*(N+1)*tiles_per_row]
+    float* seg_sum;                 // [B*(N+1)*tiles_per_row*2] float-float partition sums
+    unsigned* row_ticket;           // [B*(N+1)]
+    float* table;                   // [B*(N+1)*table_width(K)] decision tables
+    float* rhat_tail;               // [B*(N+1)*TL]
+    unsigned long long* res_best;   // [B*3]
+    unsigned* res_ticket;           // [B]
+    size_t table_smem_bytes;        // dynamic shared memory of the residual kernel
 };
 
 // Host launchers, defined next to their kernels.  dtype: 0 fp32, 1 bf16;
-// aligned: rows start on 16-byte boundaries (128-bit loads).
-cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, dim3 grid, size_t smem, cudaStream_t s);
+// tma: rows are 16-byte aligned and V * element size is a multiple of 16, so
+// tiles move with bulk copies (otherwise with plain loads).
+cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool tma, int grid, size_t smem, cudaStream_t s);
 cudaError_t launch_prune(const PruneArgs& a, int batch, size_t smem, cudaStream_t s);
-cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, dim3 stream_grid, dim3 residual_grid,
-                          cudaStream_t s);
+cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool tma, int grid, size_t smem, cudaStream_t s);
+size_t expand_smem_bytes(int max_segments, int support);
+int expand_tile_elems(int dtype);
+size_t verify_stream_smem_bytes();
+int verify_table_width(int K);
+int verify_tile_elems(int dtype);
 
 }  // namespace rheo

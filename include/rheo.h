@@ -14,8 +14,9 @@
  * as in Theorem 1).
  *
  * Ownership.  The caller allocates and owns every buffer (device memory unless
- * stated).  The library never allocates, keeps no global state, and runs
- * asynchronously on the caller's stream.  A workspace holds scratch state of
+ * stated).  The library never allocates, keeps no global state (except the
+ * static scratch array of rheo_verify_static), and runs asynchronously on the
+ * caller's stream.  A workspace holds scratch state of
  * one cycle; it must be zeroed once by rheo_workspace_init (and again after any
  * call reported an error) and must not be shared by calls that may overlap in
  * time (use one workspace per stream).
@@ -47,7 +48,7 @@ extern "C" {
 typedef struct CUstream_st* rheo_stream_t;
 
 enum { RHEO_F32 = 0, RHEO_BF16 = 1 };
-enum { RHEO_OK = 0, RHEO_EINVAL = -1, RHEO_ELAUNCH = -2 };
+enum { RHEO_OK = 0, RHEO_EINVAL = -1, RHEO_ELAUNCH = -2, RHEO_ETOOLARGE = -3 };
 
 /* device status bits */
 enum {
@@ -150,6 +151,24 @@ int rheo_verify(const rheo_config* cfg, const void* target_logits, int64_t row_s
                 const float* temperature, const uint64_t* seed, const uint64_t* offset,
                 const rheo_tree* tree, const rheo_pruned* pruned, const rheo_verify_out* out,
                 void* workspace, rheo_stream_t stream);
+
+/* Verification for callers that cannot allocate device memory where they
+ * verify (code handed only fixed input/output buffers by a host framework,
+ * runtimes whose device memory is partitioned up front, loops that must not
+ * pay cudaMalloc's implicit synchronisation).  The paper has no counterpart:
+ * this is a deployment variant of rheo_verify, same arguments and results
+ * minus the workspace.  Scratch state lives in a static device array of
+ * RHEO_STATIC_SCRATCH_BYTES that every GPU loading the library holds until
+ * exit; configurations needing more return RHEO_ETOOLARGE before any launch.
+ * The first call on a device looks the array up (make it before any stream
+ * capture).  Calls share the array: calls that overlap on the GPU race, so
+ * serialise them.  status: optional device int32 that receives this call's
+ * status word (the bits of rheo_get_status); may be NULL. */
+#define RHEO_STATIC_SCRATCH_BYTES (8u << 20)
+int rheo_verify_static(const rheo_config* cfg, const void* target_logits, int64_t row_stride,
+                       const float* temperature, const uint64_t* seed, const uint64_t* offset,
+                       const rheo_tree* tree, const rheo_pruned* pruned, const rheo_verify_out* out,
+                       int32_t* status, rheo_stream_t stream);
 
 /* Synchronise the stream, return the device status word in *status (host
  * memory) and clear it.  Returns RHEO_ELAUNCH if the stream reported an error. */

@@ -15,11 +15,12 @@ import torch
 _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "librheo.so")
 
 RHEO_F32, RHEO_BF16 = 0, 1
-RHEO_OK, RHEO_EINVAL, RHEO_ELAUNCH = 0, -1, -2
+RHEO_OK, RHEO_EINVAL, RHEO_ELAUNCH, RHEO_ETOOLARGE = 0, -1, -2, -3
 STATUS_BAD_LOGIT, STATUS_EMPTY_ROW, STATUS_BAD_TEMPERATURE, STATUS_INTERNAL = 1, 2, 4, 8
 SLOT_ROOT, SLOT_LEAD, SLOT_SAMPLED, SLOT_FILL = 0, 1, 2, 3
 
-EXPORTS = ("rheo_sizes", "rheo_workspace_init", "rheo_expand", "rheo_prune", "rheo_verify", "rheo_get_status")
+EXPORTS = ("rheo_sizes", "rheo_workspace_init", "rheo_expand", "rheo_prune", "rheo_verify", "rheo_verify_static",
+           "rheo_get_status")
 
 
 class RheoError(RuntimeError):
@@ -73,6 +74,8 @@ def lib():
         L.rheo_prune.argtypes = [C, ctypes.POINTER(_Tree), ctypes.POINTER(_Pruned), _VP, _VP]
         L.rheo_verify.argtypes = [C, _VP, ctypes.c_int64, _VP, _VP, _VP, ctypes.POINTER(_Tree),
                                   ctypes.POINTER(_Pruned), ctypes.POINTER(_VerifyOut), _VP, _VP]
+        L.rheo_verify_static.argtypes = [C, _VP, ctypes.c_int64, _VP, _VP, _VP, ctypes.POINTER(_Tree),
+                                         ctypes.POINTER(_Pruned), ctypes.POINTER(_VerifyOut), _VP, _VP]
         L.rheo_get_status.argtypes = [C, _VP, _VP, ctypes.POINTER(ctypes.c_int32)]
         for name in EXPORTS:
             getattr(L, name).restype = ctypes.c_int
@@ -241,6 +244,28 @@ def verify(cfg: Config, logits: torch.Tensor, temperature: torch.Tensor, seed: t
                              _i64(seed).data_ptr(), _i64(offset).data_ptr(), ctypes.byref(tree.c()),
                              ctypes.byref(pruned.c()), ctypes.byref(out.c()), ws.ptr(), _stream(stream)),
            "rheo_verify")
+
+
+def verify_static(cfg: Config, logits: torch.Tensor, temperature: torch.Tensor, seed: torch.Tensor,
+                  offset: torch.Tensor, tree: Tree, pruned: Pruned, out: VerifyOut,
+                  status: torch.Tensor = None, stream=None) -> None:
+    """rheo_verify_static: rheo_verify without a workspace, for callers that may
+    not allocate device memory when they verify.  Its scratch is a fixed static
+    array inside the library (calls must not overlap on the GPU); configurations
+    that need more than it holds raise RheoError with code RHEO_ETOOLARGE.
+    status: optional int32 device tensor of one element that receives the
+    call's status word."""
+    stride = _rows(cfg, logits, cfg.batch * (cfg.budget + 1))
+    st = 0
+    if status is not None:
+        if status.dtype != torch.int32 or status.numel() < 1 or not status.is_cuda:
+            raise RheoError("status must be an int32 device tensor")
+        st = status.data_ptr()
+    _check(lib().rheo_verify_static(ctypes.byref(cfg.c()), logits.data_ptr(), stride, _f32(temperature).data_ptr(),
+                                    _i64(seed).data_ptr(), _i64(offset).data_ptr(), ctypes.byref(tree.c()),
+                                    ctypes.byref(pruned.c()), ctypes.byref(out.c()), st,
+                                    _stream(stream)),
+           "rheo_verify_static")
 
 
 def status(cfg: Config, ws: Workspace, stream=None) -> int:

@@ -11,6 +11,7 @@
 #include "rheo.h"
 #include "rheo_device.cuh"
 #include "rheo_kernels.h"
+#include "stream.cuh"
 
 namespace rheo {
 namespace {
@@ -100,6 +101,11 @@ int max_segments(int64_t rows, int tpr, int grid) {
     return best;
 }
 
+// rows start on 16-byte boundaries (16-byte vector loads; a row's ragged end is read element-wise)
+bool rows_aligned(const void* p, int64_t row_stride, const rheo_config& c) {
+    return ((uintptr_t)p % 16 == 0) && ((row_stride * elem_size(c)) % 16 == 0);
+}
+
 bool tma_ok(const void* p, int64_t row_stride, const rheo_config& c) {
     const int es = elem_size(c);
     return ((uintptr_t)p % 16 == 0) && ((row_stride * es) % 16 == 0) && (((int64_t)c.vocab * es) % 16 == 0);
@@ -178,16 +184,23 @@ extern "C" int rheo_expand(const rheo_config* cfg, int32_t d, const void* logits
     a.seg_keys = at<unsigned long long>(ws, L.ex_keys);
     const int tpr = tiles_per_row(*cfg);
     const int64_t rows = (int64_t)cfg->batch * a.F;
-    // two CTAs per SM when the merge buffer of that split still fits, else one
-    int grid = (int)std::min<int64_t>(rows * tpr, 2 * (int64_t)sm_count());
-    int segs = max_segments(rows, tpr, grid);
-    size_t smem = expand_smem_bytes(segs, cfg->support);
-    if ((smem + 16 * 1024) * 2 > 227 * 1024) {
-        grid = (int)std::min<int64_t>(rows * tpr, (int64_t)sm_count());
-        segs = max_segments(rows, tpr, grid);
-        smem = expand_smem_bytes(segs, cfg->support);
+    const int sms = sm_count();
+    // Launch shape.  Up to one row per SM: every row is cut into P equal
+    // segments (P CTAs, P = SMs / rows), so a CTA holds one segment and P = 1
+    // needs no merge.  More rows: two CTAs per SM, rows cut where the even
+    // split of the tiles falls.
+    int grid;
+    if (rows <= sms) {
+        const int64_t P = std::max<int64_t>(1, std::min<int64_t>(tpr, sms / rows));
+        grid = (int)(rows * P);
+    } else {
+        grid = (int)std::min<int64_t>(rows * tpr, 2 * (int64_t)sms);
     }
-    return launch_expand(a, cfg->dtype, tma_ok(logits, row_stride, *cfg), grid, smem, (cudaStream_t)stream) ==
+    const int segs = max_segments(rows, tpr, grid);
+    a.keys_bytes = expand_keys_bytes(segs, cfg->support);
+    const size_t smem = expand_smem_bytes(segs, cfg->support);
+    if (smem + 8 * 1024 > 227 * 1024) return RHEO_EINVAL;
+    return launch_expand(a, cfg->dtype, rows_aligned(logits, row_stride, *cfg), grid, smem, (cudaStream_t)stream) ==
                    cudaSuccess
                ? RHEO_OK
                : RHEO_ELAUNCH;

@@ -1,19 +1,26 @@
 // expand.cu -- one expansion call of the draft tree (Sec. 2.1, Sec. 3.2, App. C.1).
 //
-// Persistent CTAs stream the B*F draft rows tile by tile (stream.cuh).  Over
-// each row segment a CTA keeps
+// Persistent CTAs stream the B*F draft rows in tiles of kTileBytes, each thread
+// loading its four 16-byte vectors of a tile straight into registers while it
+// still works on the previous tile; the warps never wait for one another while
+// streaming.  Over each row segment a warp keeps
 //   * a running (max, sum exp(l - max)) per thread at T = 1 (untempered, Sec. 5.4),
-//   * the segment's exact top-S keys (ord(logit) << 32 | ~id): a shared-memory
-//     candidate buffer filled with every element at or above a threshold theta
-//     that is always a lower bound of the segment's S-th key.  theta starts as
-//     a bound from the first tile (each warp's ceil(S/8)-th largest thread
-//     maximum; their minimum has >= S elements above it) and is raised to the
-//     exact S-th key whenever the buffer is compacted.
-// At the end of a segment the list and the partial sums go to the workspace.
-// The CTA that ends the last segment of a row (arrival counter, never a wait)
-// merges the lists into the row's sorted support, draws Y from the tempered
-// tail by Gumbel-max and writes the K+1 children; the last row of a request
-// selects the next frontier.
+//   * its candidate keys (ord(logit) << 32 | ~id) in a region of shared memory:
+//     every element whose key reaches theta, a lower bound of the segment's
+//     S-th key.  At the first tile theta is the minimum over warps of each
+//     warp's ceil(S/8)-th largest vector maximum; on the segment's tiles 2, 4,
+//     8, ... every warp republishes that statistic over its lanes' running
+//     vector maxima, so theta follows the S-th largest element seen so far.  A
+//     warp whose region fills up cuts it to its own S best keys, which raises
+//     theta too.  A shared 4096-bin histogram of the candidates' top key bits
+//     is kept along.
+// At the end of a segment the histogram locates the bin of the S-th key, and
+// only that bin's keys are ranked.  A row held by one CTA goes straight on to
+// its children; otherwise the lists and partial sums go to the workspace and
+// the CTA that ends the last segment of a row (arrival counter, never a wait)
+// merges them.  Then the row's sorted support gives Y from the tempered tail by
+// Gumbel-max and the K+1 children; the last row of a request selects the next
+// frontier.
 #include "rheo_device.cuh"
 #include "rheo_kernels.h"
 #include "stream.cuh"
@@ -22,210 +29,289 @@ namespace rheo {
 
 namespace {
 
-constexpr int kCand = 1024;      // candidate buffer (keys) of a segment
-constexpr int kCandHigh = 896;   // compact when the buffer holds more than this
+constexpr int kRegion = 256;   // candidate keys per warp
+constexpr int kVPT = 4;        // 16-byte vectors per thread per tile
+constexpr int kBins = 4096;    // histogram of the top 12 key bits
+constexpr int kBinShift = 52;  // key >> kBinShift is the bin
 
 struct E2Smem {
-    unsigned long long sel[kMaxSupport];
     unsigned long long sorted[kMaxSupport];
     int32_t id[kMaxSupport];
     float l[kMaxSupport];
     float lq0[kMaxSupport];
     float q[kMaxSupport];
     float lp;
-    int sel_count;
     int best;
     float lse1;
     int bad;
+};
+
+struct HistSel {
+    int bin, above, tie_n;
 };
 
 __device__ __forceinline__ unsigned long long make_key(uint32_t k32, int64_t id) {
     return ((unsigned long long)k32 << 32) | (0xFFFFFFFFu - (uint32_t)id);
 }
 
-// k-th largest (1-based) of the 32 lanes' values, all lanes get it
-__device__ __forceinline__ uint32_t warp_kth_largest(uint32_t x, int k) {
+// Cut a warp's region down to its S best keys; returns the S-th key, a lower
+// bound of the segment's S-th key.  cnt > S on entry.  The histogram loses the
+// keys that go.
+__device__ __noinline__ unsigned long long warp_cut_region(unsigned long long* region, int& cnt, int S,
+                                                           unsigned* vh) {
     const int lane = threadIdx.x & 31;
-    int rank = 0;
+    unsigned long long x[kRegion / 32];
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
-        const uint32_t y = __shfl_sync(0xFFFFFFFFu, x, j);
-        rank += (y > x) || (y == x && j < lane);
+    for (int i = 0; i < kRegion / 32; ++i) {
+        const int j = lane + 32 * i;
+        x[i] = j < cnt ? region[j] : 0ull;
     }
-    const unsigned who = __ballot_sync(0xFFFFFFFFu, rank == k - 1);
-    return __shfl_sync(0xFFFFFFFFu, x, __ffs(who) - 1);
-}
-
-// Top-`keep` of the buffer: returns the threshold T (keys >= T are kept).
-__device__ unsigned long long select_buffer(const unsigned long long* buf, int n, int keep, unsigned* hist,
-                                            RadixScratch& rs) {
-    if (n <= keep) return 1ull;
-    return block_radix_threshold([&](int i) { return buf[i]; }, n, keep, hist, rs);
-}
-
-// Keep the buffer entries >= thr (the buffer holds at most kCand keys).
-__device__ void compact_buffer(unsigned long long* buf, int n, unsigned long long thr, int* count) {
-    const int tid = threadIdx.x;
-    unsigned long long mine[kCand / kThreads];
+    const unsigned long long thr = warp_kth_largest_of<kRegion / 32>(x, S);
+    __syncwarp();
+    int w = 0;
 #pragma unroll
-    for (int j = 0; j < kCand / kThreads; ++j) {
-        const int i = tid + j * kThreads;
-        mine[j] = (i < n) ? buf[i] : 0ull;
+    for (int i = 0; i < kRegion / 32; ++i) {
+        const bool keep = x[i] != 0ull && x[i] >= thr;
+        if (x[i] != 0ull && !keep) atomicSub(&vh[(unsigned)(x[i] >> kBinShift)], 1u);
+        const unsigned bal = __ballot_sync(0xFFFFFFFFu, keep);
+        if (keep) region[w + __popc(bal & ((1u << lane) - 1u))] = x[i];
+        w += __popc(bal);
     }
-    __syncthreads();
-    if (tid == 0) *count = 0;
-    __syncthreads();
-#pragma unroll
-    for (int j = 0; j < kCand / kThreads; ++j)
-        if (mine[j] && mine[j] >= thr) buf[atomicAdd(count, 1)] = mine[j];
-    __syncthreads();
+    __syncwarp();
+    cnt = w;
+    return thr;
 }
 
-
-// Overflow of the candidate buffer while adding one tile (massive ties, or a
-// weak bound): exact S-th key of (buffer before this tile) U (tile elements >=
-// theta), read again from the tile in shared memory; keeps exactly those keys.
-template <int DT>
-__device__ __noinline__ uint32_t tile_overflow(const unsigned char* tile, int ne, int64_t e0, uint32_t theta,
-                                               unsigned long long* cand, int before, int S, int* count,
-                                               unsigned* hist, RadixScratch& rs) {
+// The tile's vectors of this thread: elements [e0 + (j*kThreads + tid)*VEC, +VEC);
+// positions at or past V read as -inf.
+template <int DT, bool ALIGNED>
+__device__ __forceinline__ void load_tile(uint4 (&v)[kVPT], const char* row, int e0, int V) {
     using E = Elem<DT>;
+    constexpr int TE = kVPT * kThreads * E::VEC;
+    if (ALIGNED && e0 + TE <= V) {  // a whole tile: plain 16-byte loads
+#pragma unroll
+        for (int j = 0; j < kVPT; ++j)
+            v[j] = ld_stream(row + ((int64_t)e0 + (j * kThreads + (int)threadIdx.x) * E::VEC) * E::SIZE);
+        return;
+    }
+#pragma unroll
+    for (int j = 0; j < kVPT; ++j)
+        v[j] = load_vec<DT, ALIGNED>(row, (int64_t)e0 + (j * kThreads + (int)threadIdx.x) * E::VEC, V);
+}
+
+// Append the keys >= thr among get(i), i < n, to sel (at most cap of them);
+// positions come from one shared counter, one atomic per warp and step.
+template <class Get>
+__device__ __forceinline__ void gather_at_least(Get get, int n, unsigned long long thr, unsigned long long* sel,
+                                                int cap, int* counter) {
+    const int lane = threadIdx.x & 31;
+    for (int i0 = 0; i0 < n; i0 += kThreads) {
+        const int i = i0 + (int)threadIdx.x;
+        const unsigned long long x = i < n ? get(i) : 0ull;
+        const bool take = x != 0ull && x >= thr;
+        const unsigned bal = __ballot_sync(0xFFFFFFFFu, take);
+        int base = 0;
+        if (lane == 0 && bal) base = atomicAdd(counter, __popc(bal));
+        base = __shfl_sync(0xFFFFFFFFu, base, 0);
+        const int pos = base + __popc(bal & ((1u << lane) - 1u));
+        if (take && pos < cap) sel[pos] = x;
+    }
+}
+
+// The k best of the distinct nonzero keys get(i), i < n, in descending order
+// into sorted[0, k); returns how many there are (min(k, number of keys)).
+// vh holds the keys' bin counts on entry; the bins that take part are left at
+// zero.  A scan of the histogram from the top gives every bin its offset in a
+// bin-ordered list; the keys of the bins down to the one holding the k-th key
+// are scattered there (tmp, tmp_cap entries) and each one is ranked among the
+// keys of its own bin only.  When that list would not fit (a huge tie class),
+// the k-th key is found by block_kth_key and the k keys are ranked directly.
+template <class Get>
+__device__ int hist_top_sorted(Get get, int n, int k, unsigned* vh, int* off, unsigned long long* tmp, int tmp_cap,
+                               unsigned long long* sorted, HistSel& hs, Red& red, int& par, unsigned* hist256,
+                               SelScratch& ss) {
+    constexpr int kPer = kBins / kThreads;
     const int tid = threadIdx.x;
-    auto elem_key = [&](int e) -> uint32_t {
-        const uint32_t raw = (DT == 0) ? reinterpret_cast<const uint32_t*>(tile)[e]
-                                       : (uint32_t)reinterpret_cast<const uint16_t*>(tile)[e];
-        return E::key(raw);
-    };
-    const unsigned long long thr = block_radix_threshold(
-        [&](int i) -> unsigned long long {
-            if (i < before) return cand[i];
-            const int e = i - before;
-            const uint32_t kk = elem_key(e);
-            return kk >= theta ? make_key(kk, e0 + e) : 0ull;
-        },
-        before + ne, S, hist, rs);
-    compact_buffer(cand, before, thr, count);
-    for (int e = tid; e < ne; e += kThreads) {
-        const uint32_t kk = elem_key(e);
-        if (kk >= theta) {
-            const unsigned long long x = make_key(kk, e0 + e);
-            if (x >= thr) cand[atomicAdd(count, 1)] = x;
+    const int hi = kBins - 1 - tid * kPer;  // this thread's bins, from the top: hi, hi-1, ...
+    unsigned c[kPer];
+    int tot = 0;
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+        c[q] = vh[hi - q];
+        tot += (int)c[q];
+    }
+    int total;
+    const int before = red_scan(tot, total, red, par);
+    const int kk = k < total ? k : total;
+    if (kk <= 0) return 0;
+    {
+        int acc = before;
+#pragma unroll
+        for (int q = 0; q < kPer; ++q) {
+            off[hi - q] = acc;
+            if (acc < kk && acc + (int)c[q] >= kk) {
+                hs.bin = hi - q;
+                hs.above = acc + (int)c[q];  // keys in the bins down to and with this one
+            }
+            acc += (int)c[q];
         }
     }
     __syncthreads();
-    return (uint32_t)(thr >> 32);
+    const int bstar = hs.bin, nsel = hs.above;
+    if (nsel <= tmp_cap) {
+        for (int i = tid; i < n; i += kThreads) {
+            const unsigned long long x = get(i);
+            const int b = (int)(x >> kBinShift);
+            if (x != 0ull && b >= bstar) tmp[off[b] + (int)atomicSub(&vh[b], 1u) - 1] = x;
+        }
+        __syncthreads();
+        for (int p = tid; p < nsel; p += kThreads) {
+            const unsigned long long x = tmp[p];
+            const int b = (int)(x >> kBinShift);
+            const int s0 = off[b], e = (b == bstar) ? nsel : off[b - 1];
+            int rank = 0;
+            for (int q = s0; q < e; ++q) rank += tmp[q] > x;
+            if (s0 + rank < kk) sorted[s0 + rank] = x;
+        }
+        __syncthreads();
+        return kk;
+    }
+    // a tie class too large for the list
+    const unsigned long long thr = block_kth_key(get, n, kk, hist256, ss);
+    if (tid == 0) hs.tie_n = 0;
+    __syncthreads();
+    gather_at_least(get, n, thr, tmp, kk, &hs.tie_n);
+    __syncthreads();
+    for (int p = tid; p < kk; p += kThreads) {
+        const unsigned long long x = tmp[p];
+        int rank = 0;
+        for (int q = 0; q < kk; ++q) rank += tmp[q] > x;
+        if (rank < kk) sorted[rank] = x;
+    }
+    __syncthreads();
+    return kk;
+}
+
+// Slow insertion path of one tile's candidates (pend: this lane's element
+// bits; the lanes' vectors are in wspill): one candidate per lane and round,
+// keys below theta dropped, the region cut to its S best whenever it fills.
+template <int DT>
+__device__ __noinline__ void insert_rounds(unsigned long long* region, int& cnt, uint32_t pend, const uint4* wspill,
+                                           int e0, unsigned long long& theta, int S, unsigned* vh,
+                                           unsigned long long* s_theta) {
+    using E = Elem<DT>;
+    constexpr int VEC = E::VEC;
+    const int lane = threadIdx.x & 31, tid = threadIdx.x;
+    const uint32_t* wv0 = reinterpret_cast<const uint32_t*>(wspill);
+    while (__any_sync(0xFFFFFFFFu, pend != 0u)) {
+        if (cnt > kRegion - 32) {
+            const unsigned long long thr = warp_cut_region(region, cnt, S, vh);
+            if (lane == 0) atomicMax(s_theta, thr);
+            theta = thr > theta ? thr : theta;
+        }
+        unsigned long long x = 0ull;
+        if (pend) {
+            const int q = __ffs(pend) - 1;
+            pend &= pend - 1u;
+            const int j = q / VEC, i = q % VEC;
+            const uint32_t* wv = wv0 + (j * 32 + lane) * 4;
+            const uint32_t raw = (DT == 0) ? wv[i] : ((wv[i >> 1] >> ((i & 1) * 16)) & 0xFFFFu);
+            x = make_key(E::key(raw), (int64_t)e0 + (j * kThreads + tid) * VEC + i);
+            if (x < theta) x = 0ull;
+        }
+        const unsigned bal = __ballot_sync(0xFFFFFFFFu, x != 0ull);
+        if (x) {
+            region[cnt + __popc(bal & ((1u << lane) - 1u))] = x;
+            atomicAdd(&vh[(unsigned)(x >> kBinShift)], 1u);
+        }
+        cnt += __popc(bal);
+    }
 }
 
 }  // namespace
 
-template <int DT, bool TMA>
+template <int DT, bool ALIGNED>
 __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a) {
     using E = Elem<DT>;
     using W = Vec<DT>;
     constexpr int VEC = E::VEC;
-    constexpr int TE = kTileBytes / E::SIZE;   // elements per tile
-    constexpr int VPT = TE / VEC / kThreads;   // 16-byte vectors per thread per tile
-    static_assert(VPT == 4, "tile layout");
+    constexpr int TE = kTileBytes / E::SIZE;  // elements per tile
+    static_assert(TE == kVPT * VEC * kThreads, "tile layout");
+    static_assert(kBins % kThreads == 0, "histogram split");
     constexpr float kLog2e = 1.4426950408889634f;
     extern __shared__ __align__(128) unsigned char dsm[];
-    unsigned char* ring = dsm;
-    unsigned long long* cand = reinterpret_cast<unsigned long long*>(dsm + kStages * kTileBytes);
-    unsigned long long* mkeys = cand + kCand;
-    __shared__ __align__(8) uint64_t full[kStages];
+    // per-warp candidate regions; after a segment's selection the same space
+    // holds the merge keys of a row and the frontier candidates of a request
+    unsigned long long* keys = reinterpret_cast<unsigned long long*>(dsm);
+    // per-warp copy of the lanes' vectors of a tile that has candidates
+    uint4* spill = reinterpret_cast<uint4*>(dsm + a.keys_bytes);
+    unsigned* vh = reinterpret_cast<unsigned*>(dsm + a.keys_bytes + sizeof(uint4) * kWarps * 32 * kVPT);
+    int* off = reinterpret_cast<int*>(vh + kBins);  // bin offsets of the top-S sort
+    // the spill area doubles as the bin-ordered list of the top-S sort
+    unsigned long long* tmpk = reinterpret_cast<unsigned long long*>(spill);
+    constexpr int kTmpCap = kWarps * 32 * kVPT * (int)sizeof(uint4) / (int)sizeof(unsigned long long);
+    __shared__ unsigned long long s_theta;
+    __shared__ uint32_t s_wb[kWarps];
+    __shared__ int s_rcount[kWarps];
     __shared__ BlockScratch bs;
+    __shared__ Red red;
     __shared__ E2Smem e2;
-    __shared__ int s_count;
-    __shared__ uint32_t s_wk[3][kWarps];
-    __shared__ int s_wtot[2][kWarps];
+    __shared__ HistSel hs;
     __shared__ unsigned s_hist[kRadixBins];
-    __shared__ RadixScratch s_rad;
+    __shared__ SelScratch s_sel;
 
     const Dims& n = a.n;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int V = n.V, S = n.S, K = n.K, m = n.m, TL = n.TL;
     const int tpr = (V + TE - 1) / TE;
+    const int kb = (S + kWarps - 1) / kWarps;  // per-warp share of S in the bounds
     const TileSplit sp{(int64_t)n.B * a.F * tpr, (int)gridDim.x};
     const int64_t t0 = sp.begin(blockIdx.x), t1 = sp.begin(blockIdx.x + 1);
-    int parity = 0;
+    unsigned long long* region = keys + warp * kRegion;
+    uint4* wspill = spill + warp * (32 * kVPT);
+    int par = 0;
 
-    if (tid == 0) {
-        s_count = 0;
-        if (TMA) {
-            for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
-            mbar_fence_init();
-        }
-    }
-    __syncthreads();
-    auto issue = [&](int64_t t) {  // thread 0: start the copy of tile t into its stage
-        const int64_t r = t / tpr;
-        const int64_t e0 = (t % tpr) * (int64_t)TE;
-        const unsigned bytes = (unsigned)(min((int64_t)TE, (int64_t)V - e0) * E::SIZE);
-        const int s = (int)((t - t0) % kStages);
-        mbar_arrive_expect_tx(&full[s], bytes);
-        bulk_load(ring + s * kTileBytes, a.logits + r * a.row_stride_bytes + e0 * E::SIZE, bytes, &full[s]);
-    };
-    int64_t issued = t0;
-    if (TMA && tid == 0)
-        for (; issued < min(t1, t0 + kStages); ++issued) issue(issued);
+    if (tid == 0) s_theta = 0ull;
 
-    // per-segment state; theta, before and seg_valid are the same in every thread
+    // per-segment state; cnt, theta and seg_valid are warp-uniform
     float mu = -INFINITY, sum = 0.0f;
-    uint32_t theta = 0;
-    int before = 0;
+    unsigned long long theta = 0ull;
+    int cnt = 0, seg_tiles = 0;
     int64_t seg_valid = 0;
-    bool timed_out = false;
-    int64_t t = t0;
-    for (; t < t1; ++t) {
-        const int64_t r = t / tpr;
-        const int tt = (int)(t % tpr);
+    int64_t r = t0 / tpr;
+    int tt = (int)(t0 % tpr);
+    uint4 nxt[kVPT];
+    if (t0 < t1) load_tile<DT, ALIGNED>(nxt, a.logits + r * a.row_stride_bytes, tt * TE, V);
+    for (int64_t t = t0; t < t1; ++t, ++tt) {
+        if (tt == tpr) {
+            tt = 0;
+            ++r;
+        }
         const bool seg_first = (t == t0) || (tt == 0);
         const bool seg_last = (t == t1 - 1) || (tt == tpr - 1);
-        const int s = (int)((t - t0) % kStages);
-        const int64_t e0 = (int64_t)tt * TE;
-        const int ne = (int)min((int64_t)TE, (int64_t)V - e0);
-        unsigned char* tile = ring + s * kTileBytes;
-        bool ok = true;
-        if (TMA) {
-            ok = mbar_wait(&full[s], (unsigned)(((t - t0) / kStages) & 1));
-        } else {
-            const char* row = a.logits + r * a.row_stride_bytes;
-            for (int e = tid; e < ne; e += kThreads) {
-                const uint32_t w = E::load_scalar(row, e0 + e);
-                if (DT == 0) reinterpret_cast<uint32_t*>(tile)[e] = w;
-                else reinterpret_cast<uint16_t*>(tile)[e] = (uint16_t)w;
-            }
-            __syncthreads();
-        }
-        const bool fullt = (ne == TE);
-        uint4 v[VPT];
+        const int e0 = tt * TE;
+        const int ne = min(TE, V - e0);
+        uint4 v[kVPT];
 #pragma unroll
-        for (int j = 0; j < VPT; ++j) {
-            v[j] = *reinterpret_cast<const uint4*>(tile + (size_t)(j * kThreads + tid) * 16);
-            if (!fullt) v[j] = W::mask(v[j], ne - (j * kThreads + tid) * VEC);
+        for (int j = 0; j < kVPT; ++j) v[j] = nxt[j];
+        if (t + 1 < t1) {  // the next tile is in flight while this one is worked on
+            const bool wrap = (tt + 1 == tpr);
+            load_tile<DT, ALIGNED>(nxt, a.logits + (r + (wrap ? 1 : 0)) * a.row_stride_bytes, wrap ? 0 : e0 + TE, V);
         }
-        float vm[VPT];
+        float vm[kVPT];
 #pragma unroll
-        for (int j = 0; j < VPT; ++j) vm[j] = W::vmax(v[j]);
+        for (int j = 0; j < kVPT; ++j) vm[j] = W::vmax(v[j]);
         const float tmax = fmaxf(fmaxf(vm[0], vm[1]), fmaxf(vm[2], vm[3]));
 
         if (seg_first) {
             mu = -INFINITY;
             sum = 0.0f;
             seg_valid = 0;
-            before = 0;
-            // bootstrap from this tile: every warp has >= kk thread maxima >= its kk-th largest
-            const uint32_t kmax = (tid * VEC < ne) ? E::key_of_value(tmax) : 0u;
-            const uint32_t w = warp_kth_largest(kmax, (S + kWarps - 1) / kWarps);
-            if (lane == 0) s_wk[0][warp] = w;
-            __syncthreads();
-            uint32_t th = s_wk[0][0];
-#pragma unroll
-            for (int i = 1; i < kWarps; ++i) th = min(th, s_wk[0][i]);
-            theta = th;
+            cnt = 0;
+            for (int i = tid; i < kBins; i += kThreads) vh[i] = 0u;
         }
-        seg_valid += ne;
-
-        // running partition sum at T = 1 (online max); mu is also the running maximum
+        // running partition sum at T = 1 (online max); mu is also the running
+        // maximum of this thread's elements
         if (tmax > mu) {
             if (mu != -INFINITY) sum *= fast_exp2((mu - tmax) * kLog2e);
             mu = tmax;
@@ -235,151 +321,168 @@ __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a)
             sum += (W::vexp(v[0], kLog2e, mc) + W::vexp(v[1], kLog2e, mc)) +
                    (W::vexp(v[2], kLog2e, mc) + W::vexp(v[3], kLog2e, mc));
         }
+        // on the segment's tiles 1, 2, 4, 8, ... this warp's bound: the kb-th
+        // largest running maximum of its lanes (lanes with no element count as
+        // absent); kb lanes hold an element at or above it
+        seg_tiles = seg_first ? 1 : seg_tiles + 1;
+        if ((seg_tiles & (seg_tiles - 1)) == 0) {
+            const uint32_t lk = (mu > -INFINITY) ? E::key_of_value(mu) : 0u;
+            int rank = 0;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                const uint32_t y = __shfl_sync(0xFFFFFFFFu, lk, j);
+                rank += (y > lk || (y == lk && j < lane)) ? 1 : 0;
+            }
+            const unsigned who = __ballot_sync(0xFFFFFFFFu, rank == kb - 1);
+            const uint32_t wb = __shfl_sync(0xFFFFFFFFu, lk, __ffs(who) - 1);
+            if (lane == 0) s_wb[warp] = wb;  // bounds only grow within a segment
+        }
+        // every warp has kb elements at or above its bound, so at least S elements
+        // reach the smallest bound (read again after a refresh, and on the tile
+        // after it, when the other warps have refreshed too)
+        if (seg_first) __syncthreads();
+        if (seg_tiles <= 2 || ((seg_tiles - 1) & (seg_tiles - 2)) == 0 || (seg_tiles & (seg_tiles - 1)) == 0) {
+            uint32_t b = *reinterpret_cast<volatile uint32_t*>(&s_wb[0]);
+#pragma unroll
+            for (int w = 1; w < kWarps; ++w) b = min(b, *reinterpret_cast<volatile uint32_t*>(&s_wb[w]));
+            const unsigned long long tb = (unsigned long long)b << 32;
+            theta = seg_first ? tb : (tb > theta ? tb : theta);
+        }
+        {
+            const unsigned long long ts = *reinterpret_cast<volatile unsigned long long*>(&s_theta);
+            theta = ts > theta ? ts : theta;
+        }
+        seg_valid += ne;
 
-        // candidates: elements >= theta (float compare; the key order is the value order)
-        const float thv = E::threshold_value(theta);
-        uint32_t cmask = 0u;
+
+        // candidates: elements whose value reaches theta's (a superset of the keys
+        // >= theta; the final selection is exact).  Every lane writes its own at
+        // offsets from a warp scan.
+        auto screen = [&](float thv) -> uint32_t {
+            uint32_t pm = 0u;
 #pragma unroll
-        for (int j = 0; j < VPT; ++j)
-            if (vm[j] >= thv)
+            for (int j = 0; j < kVPT; ++j)
+                if (vm[j] >= thv) {
+                    if (ne == TE) {
 #pragma unroll
-                for (int i = 0; i < VEC; ++i) {
-                    const float x = E::value(E::raw(v[j], i));
-                    cmask |= (x >= thv && (fullt || (j * kThreads + tid) * VEC + i < ne)) ? (1u << (j * VEC + i)) : 0u;
+                        for (int i = 0; i < VEC; ++i)
+                            pm |= (E::value(E::raw(v[j], i)) >= thv) ? (1u << (j * VEC + i)) : 0u;
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < VEC; ++i) {
+                            const bool in = (j * kThreads + tid) * VEC + i < ne;
+                            pm |= (in && E::value(E::raw(v[j], i)) >= thv) ? (1u << (j * VEC + i)) : 0u;
+                        }
+                    }
                 }
-        const int c = __popc(cmask);
-        int incl = c;
+            return pm;
+        };
+        uint32_t pend = screen(E::threshold_value((uint32_t)(theta >> 32)));
+        if (__any_sync(0xFFFFFFFFu, pend != 0u)) {
 #pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-            if (lane >= o) incl += y;
-        }
-        // next lower bound of the segment's S-th key from the running thread maxima
-        const uint32_t wk = warp_kth_largest((seg_valid > (int64_t)tid * VEC) ? E::key_of_value(mu) : 0u,
-                                             (S + kWarps - 1) / kWarps);
-        if (lane == 31) s_wtot[t & 1][warp] = incl;
-        if (lane == 0) s_wk[1 + (t & 1)][warp] = wk;
-        if (!__syncthreads_and(ok)) {  // also: every thread is done reading the stage
-            timed_out = true;
-            break;
-        }
-        int total = 0, woff = incl - c;
-        uint32_t th_next = s_wk[1 + (t & 1)][0];
+            for (int j = 0; j < kVPT; ++j) wspill[j * 32 + lane] = v[j];
+            const int c = __popc(pend);
+            int incl = c;
 #pragma unroll
-        for (int w = 0; w < kWarps; ++w) {
-            const int x = s_wtot[t & 1][w];
-            woff += (w < warp) ? x : 0;
-            total += x;
-            th_next = min(th_next, s_wk[1 + (t & 1)][w]);
-        }
-        if (before + total <= kCand) {
-            int pos = before + woff;
-            for (uint32_t mm = cmask; mm; mm &= mm - 1) {
-                const int q = __ffs(mm) - 1;
-                const int j = q / VEC, i = q % VEC;
-                cand[pos++] = make_key(E::key(E::raw(v[j], i)), e0 + (j * kThreads + tid) * VEC + i);
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+                if (lane >= o) incl += y;
             }
-            before += total;
-            if (TMA && tid == 0 && issued < t1) issue(issued++);
-            if (before > kCandHigh) {
-                __syncthreads();
-                const unsigned long long thr = select_buffer(cand, before, S, s_hist, s_rad);
-                compact_buffer(cand, before, thr, &s_count);
-                before = s_count;
-                theta = max(theta, (uint32_t)(thr >> 32));
-                __syncthreads();
+            const int total = __shfl_sync(0xFFFFFFFFu, incl, 31);
+            if (cnt + total <= kRegion) {
+                const uint32_t* wv0 = reinterpret_cast<const uint32_t*>(wspill);
+                int pos = cnt + incl - c;
+                for (uint32_t mm = pend; mm; mm &= mm - 1u) {
+                    const int q = __ffs(mm) - 1;
+                    const int j = q / VEC, i = q % VEC;
+                    const uint32_t* wv = wv0 + (j * 32 + lane) * 4;
+                    const uint32_t raw = (DT == 0) ? wv[i] : ((wv[i >> 1] >> ((i & 1) * 16)) & 0xFFFFu);
+                    const unsigned long long x = make_key(E::key(raw), (int64_t)e0 + (j * kThreads + tid) * VEC + i);
+                    region[pos++] = x;
+                    atomicAdd(&vh[(unsigned)(x >> kBinShift)], 1u);
+                }
+                cnt += total;
+            } else {
+                // the region would overflow: one candidate per lane and round,
+                // keys below theta dropped, the region cut whenever it fills
+                insert_rounds<DT>(region, cnt, pend, wspill, e0, theta, S, vh, &s_theta);
             }
-        } else {
-            // overflow (massive ties, or a weak bound): rebuild from the tile, which
-            // stays in shared memory until this is done
-            __syncthreads();
-            theta = tile_overflow<DT>(tile, ne, e0, theta, cand, before, S, &s_count, s_hist, s_rad);
-            before = s_count;
-            __syncthreads();
-            if (TMA && tid == 0 && issued < t1) issue(issued++);
+            __syncwarp();
         }
-        theta = max(theta, th_next);
-
         if (!seg_last) continue;
-        __syncthreads();  // the candidate writes of this tile are visible
-        const int cnt = before;
 
-        // ---- end of segment: exact top-S list and partial sums to the workspace ----
+        // ---- end of segment: exact top-S keys ------------------------------------
+        if (lane == 0) s_rcount[warp] = cnt;
+        float Ms;
+        const FF Ss = red_partition(mu, sum, kLog2e, Ms, red, par);  // its barrier also publishes the counts
+        if (tid == 0) s_theta = 0ull;  // every warp is past its last cut: ready for the next segment
         const int target = (int)min((int64_t)S, seg_valid);
-        const unsigned long long thr = select_buffer(cand, cnt, target, s_hist, s_rad);
+        auto rkey = [&](int i) -> unsigned long long {
+            return (i % kRegion) < s_rcount[i / kRegion] ? keys[i] : 0ull;
+        };
+        const int written = hist_top_sorted(rkey, kWarps * kRegion, target, vh, off, tmpk, kTmpCap, e2.sorted, hs,
+                                            red, par, s_hist, s_sel);
         const int first_owner = sp.owner(r * tpr);
         const int seg = (int)blockIdx.x - first_owner;
         const int nseg = sp.owner(r * tpr + tpr - 1) - first_owner + 1;
-        unsigned long long* out = a.seg_keys + ((int64_t)r * tpr + seg) * S;
-        __syncthreads();
-        if (tid == 0) e2.sel_count = 0;
-        __syncthreads();
-        for (int i = tid; i < cnt; i += kThreads)
-            if (cand[i] >= thr) {
-                const int pos = atomicAdd(&e2.sel_count, 1);
-                if (pos < S) out[pos] = cand[i];
-            }
-        const float Ms = block_max_f32(mu, bs);
-        const FF Ss = block_sum_ff((mu != -INFINITY) ? sum * fast_exp2((mu - Ms) * kLog2e) : sum, bs);
-        const int written = e2.sel_count;
-        for (int i = written + tid; i < S; i += kThreads) out[i] = 0ull;
+        const int b = (int)(r / a.F), f = (int)(r % a.F);
         if (tid == 0) {
-            a.seg_mu[(int64_t)r * tpr + seg] = Ms;
-            a.seg_sum[2 * ((int64_t)r * tpr + seg)] = Ss.hi;
-            a.seg_sum[2 * ((int64_t)r * tpr + seg) + 1] = Ss.lo;
             if (isnan(Ss.hi) || Ms == INFINITY) atomicOr(a.status, kStBadLogit);
             if (written != target) atomicOr(a.status, kStInternal);
         }
-        if (!arrive_last(a.row_ticket + r, (unsigned)nseg, bs)) continue;
+        if (nseg == 1) {
+            // the whole row is here: its support is e2.sorted, its partition sum Ss
+            if (tid == 0) {
+                const FF l = ff_add(ff_log(Ss), Ms);
+                e2.lse1 = __fadd_rn(l.hi, l.lo);
+                e2.bad = (written != S) ? 1 : 0;
+            }
+        } else {
+            unsigned long long* out = a.seg_keys + ((int64_t)r * tpr + seg) * S;
+            for (int i = tid; i < S; i += kThreads) out[i] = i < written ? e2.sorted[i] : 0ull;
+            if (tid == 0) {
+                a.seg_mu[(int64_t)r * tpr + seg] = Ms;
+                a.seg_sum[2 * ((int64_t)r * tpr + seg)] = Ss.hi;
+                a.seg_sum[2 * ((int64_t)r * tpr + seg) + 1] = Ss.lo;
+            }
+            if (!arrive_last(a.row_ticket + r, (unsigned)nseg, bs)) continue;
 
-        // ---- last segment of row r: support, tail sample, pool ---------------------
-        const int b = (int)(r / a.F), f = (int)(r % a.F);
-        const int nkeys = nseg * S;
-        const unsigned long long* rk = a.seg_keys + (int64_t)r * tpr * S;
-        for (int i = tid; i < nkeys; i += kThreads) mkeys[i] = __ldcg(rk + i);
-        __syncthreads();
-        {
-            int nz = 0;
-            for (int i = tid; i < nkeys; i += kThreads) nz += mkeys[i] != 0ull;
-            nz = block_sum_int(nz, bs, parity);
-            unsigned long long rthr = 1ull;
-            if (nz > S) rthr = block_radix_threshold([&](int i) { return mkeys[i]; }, nkeys, S, s_hist, s_rad);
-            if (tid == 0) e2.sel_count = 0;
+            // ---- last segment of row r: merge the segments' lists and sums ---------
+            const int nkeys = nseg * S;
+            const unsigned long long* rk = a.seg_keys + (int64_t)r * tpr * S;
+            for (int i = tid; i < kBins; i += kThreads) vh[i] = 0u;
             __syncthreads();
             for (int i = tid; i < nkeys; i += kThreads) {
-                const unsigned long long x = mkeys[i];
-                if (x && x >= rthr) {
-                    const int pos = atomicAdd(&e2.sel_count, 1);
-                    if (pos < S) e2.sel[pos] = x;
+                const unsigned long long x = __ldcg(rk + i);
+                keys[i] = x;
+                if (x) atomicAdd(&vh[(unsigned)(x >> kBinShift)], 1u);
+            }
+            __syncthreads();
+            const int got = hist_top_sorted([&](int i) { return keys[i]; }, nkeys, S, vh, off, tmpk, kTmpCap,
+                                            e2.sorted, hs, red, par, s_hist, s_sel);
+            if (tid < 32) {
+                float mx = -INFINITY;
+                for (int c = tid; c < nseg; c += 32) mx = fmaxf(mx, __ldcg(a.seg_mu + (int64_t)r * tpr + c));
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
+                FF acc{0.0f, 0.0f};
+                for (int c = tid; c < nseg; c += 32) {
+                    const int64_t q = (int64_t)r * tpr + c;
+                    const FF sc{__ldcg(a.seg_sum + 2 * q), __ldcg(a.seg_sum + 2 * q + 1)};
+                    if (sc.hi != 0.0f) acc = ff_add(acc, ff_mul(expf(__ldcg(a.seg_mu + q) - mx), sc));
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) acc = ff_add(acc, ff_shfl_xor(acc, o));
+                if (tid == 0) {
+                    const FF l = ff_add(ff_log(acc), mx);
+                    e2.lse1 = __fadd_rn(l.hi, l.lo);
                 }
             }
+            __syncthreads();
+            if (tid == 0) e2.bad = (got != S) ? 1 : 0;
         }
         __syncthreads();
-        if (tid < S) {
-            const unsigned long long x = e2.sel[tid];
-            int rank = 0;
-            for (int j = 0; j < S; ++j) rank += e2.sel[j] > x;
-            e2.sorted[rank] = x;
-        }
-        if (tid < 32) {
-            float mx = -INFINITY;
-            for (int c = tid; c < nseg; c += 32) mx = fmaxf(mx, __ldcg(a.seg_mu + (int64_t)r * tpr + c));
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
-            FF acc{0.0f, 0.0f};
-            for (int c = tid; c < nseg; c += 32) {
-                const int64_t q = (int64_t)r * tpr + c;
-                const FF sc{__ldcg(a.seg_sum + 2 * q), __ldcg(a.seg_sum + 2 * q + 1)};
-                if (sc.hi != 0.0f) acc = ff_add(acc, ff_mul(expf(__ldcg(a.seg_mu + q) - mx), sc));
-            }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) acc = ff_add(acc, ff_shfl_xor(acc, o));
-            if (tid == 0) {
-                const FF l = ff_add(ff_log(acc), mx);
-                e2.lse1 = __fadd_rn(l.hi, l.lo);
-                e2.bad = (e2.sel_count != S) ? 1 : 0;
-            }
-        }
+
         __syncthreads();
         const float lse1 = e2.lse1;
         if (tid < S) {
@@ -394,27 +497,27 @@ __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a)
         const float T = a.T[b];
         const uint64_t seed = a.seed[b], off = a.offset[b];
         const int64_t nb = (int64_t)b * n.G1;
-        int64_t par = (a.d == 1) ? 0 : (int64_t)a.tree.frontier[(int64_t)b * K + f];
-        if (par < 0 || par >= n.G1) {  // frontier never written for this tree
+        int64_t par_g = (a.d == 1) ? 0 : (int64_t)a.tree.frontier[(int64_t)b * K + f];
+        if (par_g < 0 || par_g >= n.G1) {  // frontier never written for this tree
             if (tid == 0) atomicOr(a.status, kStInternal);
-            par = 0;
+            par_g = 0;
         }
         const int64_t eidx = (a.d == 1) ? 0 : 1 + (int64_t)(a.d - 2) * K + f;
         const int64_t g0 = depth_base(K, a.d) + (int64_t)f * (K + 1);
 
         // tempered tail q~ = softmax(l / T) over support ranks m+1..S; Y by Gumbel-max
         const float tau = (tid < TL) ? __fdiv_rn(e2.l[m + tid], T) : -INFINITY;
-        const float mt = block_max_f32(tau, bs);
-        const FF st = block_sum_ff((tid < TL && mt > -INFINITY) ? expf(tau - mt) : 0.0f, bs);
+        const float mt = __fdiv_rn(e2.l[m], T);  // the support is sorted: rank m is the tail's maximum
+        const FF st = red_sum_ff(FF{(tid < TL && mt > -INFINITY) ? expf(tau - mt) : 0.0f, 0.0f}, red, par);
         const FF lse_tail = ff_add(ff_log(st), mt);
         unsigned long long pack = 0ull;
         if (tid < TL) {
             e2.q[tid] = expf(__fsub_rn(tau, lse_tail.hi) - lse_tail.lo);
-            const float g = gumbel(uniform(seed, off, kTagSample, (int)par, (uint64_t)tid));
+            const float g = gumbel(uniform(seed, off, kTagSample, (int)par_g, (uint64_t)tid));
             const float key = __fadd_rn(tau, g);
             if (key > -INFINITY) pack = make_key(ord_f32(key), tid);
         }
-        const unsigned long long bestp = block_max_u64(pack, bs);
+        const unsigned long long bestp = red_max_u64(pack, red, par);
         if (tid == 0) {
             e2.best = bestp ? (int)(0xFFFFFFFFu - (uint32_t)bestp) : 0;
             if (e2.bad) atomicOr(a.status, kStInternal);
@@ -462,10 +565,10 @@ __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a)
                 const int qf = j - m - 1;
                 rank = m + qf + (qf >= best ? 1 : 0); lpj = e2.lq0[rank]; st8 = kSlotFill;
             }
-            const float ps = (a.d == 1) ? 0.0f : a.tree.score[nb + par];
+            const float ps = (a.d == 1) ? 0.0f : a.tree.score[nb + par_g];
             const int64_t g = nb + g0 + j;
             a.tree.token[g] = e2.id[rank];
-            a.tree.parent[g] = (int32_t)par;
+            a.tree.parent[g] = (int32_t)par_g;
             a.tree.log_proxy[g] = lpj;
             a.tree.score[g] = __fadd_rn(ps, lpj);
             a.tree.qtilde[g] = qv;
@@ -484,55 +587,62 @@ __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a)
         {
             const int nn = a.F * (K + 1);
             const int64_t base = depth_base(K, a.d);
-            const bool staged = nn <= kCand;
-            auto key_at = [&](int i) -> unsigned long long {
-                return staged ? cand[i] : make_key(ord_f32(__ldcg(a.tree.score + nb + base + i)), base + i);
-            };
-            if (staged)
-                for (int i = tid; i < nn; i += kThreads)
-                    cand[i] = make_key(ord_f32(__ldcg(a.tree.score + nb + base + i)), base + i);
-            __syncthreads();
-            const unsigned long long fthr = block_radix_threshold([&](int i) { return key_at(i); }, nn, K, s_hist, s_rad);
-            const int per = (nn + kThreads - 1) / kThreads;
-            const int lo = min(nn, tid * per), hi = min(nn, lo + per);
-            int c = 0;
-            for (int i = lo; i < hi; ++i) c += key_at(i) >= fthr;
-            int total;
-            int pos = block_exclusive_scan(c, total, bs);
-            for (int i = lo; i < hi; ++i)
-                if (key_at(i) >= fthr) {
-                    if (pos < K) a.tree.frontier[(int64_t)b * K + pos] = (int32_t)(base + i);
-                    ++pos;
-                }
-            if (tid == 0 && total != K) atomicOr(a.status, kStInternal);
+            if (nn <= kThreads) {
+                // rank of every candidate; the K best, written in gen-id order
+                const unsigned long long x =
+                    tid < nn ? make_key(ord_f32(__ldcg(a.tree.score + nb + base + tid)), base + tid) : 0ull;
+                if (tid < nn) keys[tid] = x;
+                __syncthreads();
+                int rank = 0;
+                if (tid < nn)
+                    for (int j = 0; j < nn; ++j) rank += keys[j] > x;
+                const bool take = tid < nn && rank < K;
+                int total;
+                const int pos = red_scan(take ? 1 : 0, total, red, par);
+                if (take && pos < K) a.tree.frontier[(int64_t)b * K + pos] = (int32_t)(base + tid);
+                if (tid == 0 && total != K) atomicOr(a.status, kStInternal);
+            } else {
+                auto key_at = [&](int i) -> unsigned long long {
+                    return make_key(ord_f32(__ldcg(a.tree.score + nb + base + i)), base + i);
+                };
+                const unsigned long long fthr = block_kth_key(key_at, nn, K, s_hist, s_sel);
+                const int per = (nn + kThreads - 1) / kThreads;
+                const int lo = min(nn, tid * per), hi = min(nn, lo + per);
+                int c = 0;
+                for (int i = lo; i < hi; ++i) c += key_at(i) >= fthr;
+                int total;
+                int pos = red_scan(c, total, red, par);
+                for (int i = lo; i < hi; ++i)
+                    if (key_at(i) >= fthr) {
+                        if (pos < K) a.tree.frontier[(int64_t)b * K + pos] = (int32_t)(base + i);
+                        ++pos;
+                    }
+                if (tid == 0 && total != K) atomicOr(a.status, kStInternal);
+            }
             __syncthreads();
         }
-    }
-
-    if (timed_out) {
-        if (tid == 0) {
-            atomicOr(a.status, kStTimeout);
-            // let the copies still in flight land before the CTA leaves
-            for (int64_t u = t; u < issued; ++u)
-                mbar_wait(&full[(int)((u - t0) % kStages)], (unsigned)(((u - t0) / kStages) & 1));
-        }
-        __syncthreads();
     }
 }
 
-cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool tma, int grid, size_t smem, cudaStream_t s) {
+cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, int grid, size_t smem, cudaStream_t s) {
     auto go = [&](auto kern) {
         cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (err != cudaSuccess) return err;
         kern<<<grid, kThreads, smem, s>>>(a);
         return cudaGetLastError();
     };
-    if (dtype == 1) return tma ? go(expand_kernel<1, true>) : go(expand_kernel<1, false>);
-    return tma ? go(expand_kernel<0, true>) : go(expand_kernel<0, false>);
+    if (dtype == 1) return aligned ? go(expand_kernel<1, true>) : go(expand_kernel<1, false>);
+    return aligned ? go(expand_kernel<0, true>) : go(expand_kernel<0, false>);
+}
+
+size_t expand_keys_bytes(int max_segments, int support) {
+    size_t keys = (size_t)kWarps * kRegion;
+    if ((size_t)max_segments * support > keys) keys = (size_t)max_segments * support;
+    return (sizeof(unsigned long long) * keys + 127) & ~(size_t)127;  // the spill area after it is 16-byte aligned
 }
 
 size_t expand_smem_bytes(int max_segments, int support) {
-    return (size_t)kStages * kTileBytes + sizeof(unsigned long long) * (kCand + (size_t)max_segments * support);
+    return expand_keys_bytes(max_segments, support) + sizeof(uint4) * kWarps * 32 * kVPT + 2 * sizeof(unsigned) * kBins;
 }
 
 int expand_tile_elems(int dtype) { return kTileBytes / (dtype == 1 ? 2 : 4); }

@@ -364,6 +364,131 @@ __device__ __forceinline__ FF block_sum_ff(FF v, BlockScratch& s) {
 }
 __device__ __forceinline__ FF block_sum_ff(float v, BlockScratch& s) { return block_sum_ff(FF{v, 0.0f}, s); }
 
+// ---------------------------------------------------------------------------
+// Block reductions with one barrier each: the warp partials go to one of two
+// scratch buffers, alternated by the caller's parity bit, so a warp that runs
+// ahead into the next reduction never overwrites partials still being read.
+// ---------------------------------------------------------------------------
+struct Red {
+    float f[2][kWarps];
+    float g[2][kWarps];
+    unsigned long long u[2][kWarps];
+    int i[2][kWarps];
+};
+
+__device__ __forceinline__ float red_max_f32(float v, Red& r, int& par) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+    float* buf = r.f[par];
+    par ^= 1;
+    if ((threadIdx.x & 31) == 0) buf[threadIdx.x >> 5] = v;
+    __syncthreads();
+    float m = buf[0];
+#pragma unroll
+    for (int w = 1; w < kWarps; ++w) m = fmaxf(m, buf[w]);
+    return m;
+}
+
+__device__ __forceinline__ FF red_sum_ff(FF v, Red& r, int& par) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = ff_add(v, ff_shfl_xor(v, o));
+    float* bh = r.f[par];
+    float* bl = r.g[par];
+    par ^= 1;
+    if ((threadIdx.x & 31) == 0) {
+        bh[threadIdx.x >> 5] = v.hi;
+        bl[threadIdx.x >> 5] = v.lo;
+    }
+    __syncthreads();
+    FF t{bh[0], bl[0]};
+#pragma unroll
+    for (int w = 1; w < kWarps; ++w) t = ff_add(t, FF{bh[w], bl[w]});
+    return t;
+}
+
+__device__ __forceinline__ unsigned long long red_max_u64(unsigned long long v, Red& r, int& par) {
+    v = warp_max_u64(v);
+    unsigned long long* buf = r.u[par];
+    par ^= 1;
+    if ((threadIdx.x & 31) == 0) buf[threadIdx.x >> 5] = v;
+    __syncthreads();
+    unsigned long long t = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) t = buf[w] > t ? buf[w] : t;
+    return t;
+}
+
+__device__ __forceinline__ int red_sum_int(int v, Red& r, int& par) {
+    v = __reduce_add_sync(0xFFFFFFFFu, v);
+    int* buf = r.i[par];
+    par ^= 1;
+    if ((threadIdx.x & 31) == 0) buf[threadIdx.x >> 5] = v;
+    __syncthreads();
+    int t = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) t += buf[w];
+    return t;
+}
+
+// exclusive prefix sum in thread order; total in `total`
+__device__ __forceinline__ int red_scan(int v, int& total, Red& r, int& par) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+        if (lane >= o) x += y;
+    }
+    int* buf = r.i[par];
+    par ^= 1;
+    if (lane == 31) buf[warp] = x;
+    __syncthreads();
+    int before = 0;
+    total = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+        before += (w < warp) ? buf[w] : 0;
+        total += buf[w];
+    }
+    return before + x - v;
+}
+
+// Partition sum of a block: every thread holds (m, s) = (its maximum, sum of
+// 2^((x - m) c) over its values; m = -inf when it has none).  Returns
+// M = max over the block and the sum rescaled to M as float-float.
+__device__ __forceinline__ FF red_partition(float m, float s, float c, float& M, Red& r, int& par) {
+    FF v{s, 0.0f};
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o);
+        const FF v2 = ff_shfl_xor(v, o);
+        const float mm = fmaxf(m, m2);
+        const FF a = (m == -INFINITY) ? FF{0.0f, 0.0f} : ff_mul(fast_exp2((m - mm) * c), v);
+        const FF b = (m2 == -INFINITY) ? FF{0.0f, 0.0f} : ff_mul(fast_exp2((m2 - mm) * c), v2);
+        v = ff_add(a, b);
+        m = mm;
+    }
+    float* bm = r.f[par];
+    float* bh = r.g[par];
+    unsigned long long* bl = r.u[par];
+    par ^= 1;
+    if ((threadIdx.x & 31) == 0) {
+        bm[threadIdx.x >> 5] = m;
+        bh[threadIdx.x >> 5] = v.hi;
+        bl[threadIdx.x >> 5] = (unsigned long long)__float_as_uint(v.lo);
+    }
+    __syncthreads();
+    M = bm[0];
+#pragma unroll
+    for (int w = 1; w < kWarps; ++w) M = fmaxf(M, bm[w]);
+    FF t{0.0f, 0.0f};
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w)
+        if (bm[w] != -INFINITY)
+            t = ff_add(t, ff_mul(fast_exp2((bm[w] - M) * c), FF{bh[w], __uint_as_float((uint32_t)bl[w])}));
+    return t;
+}
+
 // exp(l / T - c) for an fp32 logit l and a float-float constant c, to a few
 // fp32 ulps: l / T = tau + rem / T exactly (tau correctly rounded).
 __device__ __forceinline__ float exp_scaled_minus(float l, float T, FF c) {
@@ -426,6 +551,7 @@ __device__ unsigned long long block_radix_threshold(Get get, int n, int k, unsig
         const int shift = top - bits;
         const unsigned mask = (1u << bits) - 1u;
         hist[tid] = 0u;  // kThreads == kRadixBins
+        if (tid == 0) rs.digit = -1;
         __syncthreads();
         for (int i = tid; i < n; i += kThreads) {
             const unsigned long long x = get(i);
@@ -454,6 +580,10 @@ __device__ unsigned long long block_radix_threshold(Get get, int n, int k, unsig
         }
         __syncthreads();
         const int dd = rs.digit;
+        if (dd < 0 || dd >= kRadixBins) {  // fewer keys than k (broken input): keep every key
+            __syncthreads();
+            return 1ull;
+        }
         above = rs.above;
         prefix |= (unsigned long long)dd << shift;
         const bool exact = above + (int)hist[dd] == k;
@@ -462,6 +592,182 @@ __device__ unsigned long long block_radix_threshold(Get get, int n, int k, unsig
         if (exact) break;
     }
     return prefix;
+}
+
+// ---------------------------------------------------------------------------
+// k-th largest of up to N values per lane across one warp (0 = "no value"):
+// built bit by bit from the most significant bit on, visiting only the bits in
+// which the values differ (bits common to all of them come from their AND).
+// Returns 0 when the warp holds fewer than k values.  All lanes get the result.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t warp_and_u32(uint32_t x) { return __reduce_and_sync(0xFFFFFFFFu, x); }
+__device__ __forceinline__ uint32_t warp_or_u32(uint32_t x) { return __reduce_or_sync(0xFFFFFFFFu, x); }
+__device__ __forceinline__ unsigned long long warp_and(unsigned long long x) {
+    return ((unsigned long long)warp_and_u32((uint32_t)(x >> 32)) << 32) | warp_and_u32((uint32_t)x);
+}
+__device__ __forceinline__ unsigned long long warp_or(unsigned long long x) {
+    return ((unsigned long long)warp_or_u32((uint32_t)(x >> 32)) << 32) | warp_or_u32((uint32_t)x);
+}
+__device__ __forceinline__ uint32_t warp_and(uint32_t x) { return warp_and_u32(x); }
+__device__ __forceinline__ uint32_t warp_or(uint32_t x) { return warp_or_u32(x); }
+
+template <int N, class T>
+__device__ __forceinline__ T warp_kth_largest_of(const T (&x)[N], int k) {
+    T a = ~T(0), o = T(0);
+    int c = 0;
+#pragma unroll
+    for (int i = 0; i < N; ++i)
+        if (x[i]) {
+            a &= x[i];
+            o |= x[i];
+            ++c;
+        }
+    c = __reduce_add_sync(0xFFFFFFFFu, c);
+    if (c < k) return T(0);
+    a = warp_and(a);
+    o = warp_or(o);
+    T prefix = a;
+    for (T diff = a ^ o; diff;) {
+        const int bit = (int)(sizeof(T) * 8 - 1) - (sizeof(T) == 8 ? __clzll((long long)diff) : __clz((int)diff));
+        const T b = T(1) << bit;
+        diff ^= b;
+        const T cand = prefix | b;
+        int q = 0;
+#pragma unroll
+        for (int i = 0; i < N; ++i) q += (x[i] >= cand) ? 1 : 0;
+        if (__reduce_add_sync(0xFFFFFFFFu, q) >= k) prefix = cand;
+    }
+    return prefix;
+}
+
+// ---------------------------------------------------------------------------
+// Block-wide k-th largest of n distinct nonzero 64-bit keys (get(i) == 0 means
+// "no key"; i visited as tid + j * kThreads), 1 <= k <= number of keys.  The
+// returned threshold T has exactly k keys >= T.  Rounds over the keys still in
+// play ("live": equal to the prefix found so far above bit `top`): bits common
+// to every live key are taken from their AND at once, the next 8 differing
+// bits are counted in a shared histogram and scanned from the top; a round
+// ends early when the keys at or above the prefix number exactly k, and a tie
+// class of at most 32 keys is finished by one warp ranking it.
+// ---------------------------------------------------------------------------
+struct SelScratch {
+    unsigned long long red_and[kWarps], red_or[kWarps];
+    int wsum[kWarps];
+    int digit, above, tie_n;
+    unsigned long long result;
+    unsigned long long tie[32];
+};
+
+template <class Get>
+__device__ unsigned long long block_kth_key(Get get, int n, int k, unsigned* hist, SelScratch& ss) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    unsigned long long prefix = 0ull;
+    int top = 64, above = 0;
+    auto live = [&](unsigned long long x) -> bool {
+        return x != 0ull && (top >= 64 || (x >> top) == (prefix >> top));
+    };
+    for (;;) {
+        // common bits of the live keys; the histogram is cleared meanwhile
+        unsigned long long a_and = ~0ull, a_or = 0ull;
+        int nl = 0;
+        for (int i = tid; i < n; i += kThreads) {
+            const unsigned long long x = get(i);
+            if (live(x)) {
+                a_and &= x;
+                a_or |= x;
+                ++nl;
+            }
+        }
+        a_and = warp_and(a_and);
+        a_or = warp_or(a_or);
+        nl = __reduce_add_sync(0xFFFFFFFFu, nl);
+        if (lane == 0) {
+            ss.red_and[warp] = a_and;
+            ss.red_or[warp] = a_or;
+            ss.wsum[warp] = nl;
+        }
+        hist[tid] = 0u;  // kThreads == kRadixBins
+        if (tid == 0) ss.digit = -1;
+        __syncthreads();
+        a_and = ~0ull;
+        a_or = 0ull;
+        nl = 0;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) {
+            a_and &= ss.red_and[w];
+            a_or |= ss.red_or[w];
+            nl += ss.wsum[w];
+        }
+        if (nl == 0 || above + nl < k) {  // fewer keys than k (broken input): keep every key
+            __syncthreads();
+            return 1ull;
+        }
+        const unsigned long long diff = a_and ^ a_or;
+        if (diff == 0ull) {  // a single live key: the k-th
+            __syncthreads();
+            return a_and;
+        }
+        top = 64 - __clzll((long long)diff);
+        prefix = (top >= 64) ? 0ull : (a_and >> top) << top;
+        const int bits = top >= 8 ? 8 : top;
+        const int shift = top - bits;
+        const unsigned mask = (1u << bits) - 1u;
+        for (int i = tid; i < n; i += kThreads) {
+            const unsigned long long x = get(i);
+            if (live(x)) atomicAdd(&hist[(unsigned)(x >> shift) & mask], 1u);
+        }
+        __syncthreads();
+        // thread t owns digit 255 - t: digits in descending order
+        const int d = kRadixBins - 1 - tid;
+        const int h = (int)hist[d];
+        int incl = h;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        if (lane == 31) ss.wsum[warp] = incl;
+        __syncthreads();
+        int before = above + incl - h;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) before += (w < warp) ? ss.wsum[w] : 0;
+        if (h > 0 && before < k && before + h >= k) {
+            ss.digit = d;
+            ss.above = before;
+            ss.tie_n = 0;
+        }
+        __syncthreads();
+        const int dd = ss.digit;
+        if (dd < 0) {  // cannot happen when the keys number at least k
+            __syncthreads();
+            return 1ull;
+        }
+        above = ss.above;
+        const int cnt = (int)hist[dd];
+        prefix |= (unsigned long long)dd << shift;
+        top = shift;
+        if (above + cnt == k) {
+            __syncthreads();
+            return prefix;
+        }
+        if (cnt <= 32) {  // finish the tie class in one warp
+            for (int i = tid; i < n; i += kThreads) {
+                const unsigned long long x = get(i);
+                if (live(x)) ss.tie[atomicAdd(&ss.tie_n, 1)] = x;
+            }
+            __syncthreads();
+            if (warp == 0) {
+                const unsigned long long x = lane < cnt ? ss.tie[lane] : 0ull;
+                int rank = 0;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) rank += (__shfl_sync(0xFFFFFFFFu, x, j) > x) ? 1 : 0;
+                if (x && rank == k - above - 1) ss.result = x;
+            }
+            __syncthreads();
+            return ss.result;
+        }
+        __syncthreads();  // hist and ss read by everyone before the next round
+    }
 }
 
 // exclusive prefix sum over the block (in thread order)

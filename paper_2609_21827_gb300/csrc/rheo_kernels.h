@@ -41,6 +41,7 @@ struct Dims {
 struct ExpandArgs {
     Dims n;
     int d, F;
+    size_t keys_bytes;              // dynamic shared memory for keys; the spill area follows
     const char* logits;
     int64_t row_stride_bytes;
     const float* T;
@@ -93,6 +94,7 @@ struct VerifyArgs {
 cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool tma, int grid, size_t smem, cudaStream_t s);
 cudaError_t launch_prune(const PruneArgs& a, int batch, size_t smem, cudaStream_t s);
 cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool tma, int grid, size_t smem, cudaStream_t s);
+size_t expand_keys_bytes(int max_segments, int support);
 size_t expand_smem_bytes(int max_segments, int support);
 int expand_tile_elems(int dtype);
 size_t verify_stream_smem_bytes();

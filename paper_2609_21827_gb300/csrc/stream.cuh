@@ -18,7 +18,8 @@
 namespace rheo {
 
 constexpr int kTileBytes = 16384;
-constexpr int kStages = 4;
+constexpr int kStages = 4;     // ring depth of kernels with two CTAs per SM
+constexpr int kMaxStages = 8;  // deepest ring (one CTA per SM)
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s: a copy that never lands is an error
 constexpr uint32_t kStTimeout = 16u;
 

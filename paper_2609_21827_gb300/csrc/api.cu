@@ -11,7 +11,6 @@
 #include "rheo.h"
 #include "rheo_device.cuh"
 #include "rheo_kernels.h"
-#include "stream.cuh"
 
 namespace rheo {
 namespace {
@@ -44,7 +43,7 @@ bool valid(const rheo_config* c) {
 
 struct Layout {
     size_t status, ex_row_ticket, ex_req_ticket, ex_mu, ex_sum, ex_keys;
-    size_t v_mu, v_sum, v_row_ticket, v_table, v_rhat, r_best, r_ticket;
+    size_t v_mu, v_sum, v_table, v_rhat, r_best, r_ticket;
     size_t total;
 };
 
@@ -53,6 +52,7 @@ size_t up(size_t x) { return (x + 255) & ~(size_t)255; }
 Layout layout(const rheo_config& c) {
     const int64_t B = c.batch, F = c.K > 0 ? c.K : 1, P = tiles_per_row(c), S = c.support;
     const int64_t NP = c.budget + 1, TL = c.support - c.m;
+    const int64_t VC = verify_chunks_per_row(c.dtype == RHEO_BF16 ? 1 : 0, c.vocab);
     Layout L{};
     size_t o = 0;
     auto take = [&](size_t bytes) { size_t at = o; o = up(o + bytes); return at; };
@@ -62,9 +62,8 @@ Layout layout(const rheo_config& c) {
     L.ex_mu = take(sizeof(float) * B * F * P);
     L.ex_sum = take(2 * sizeof(float) * B * F * P);
     L.ex_keys = take(sizeof(unsigned long long) * B * F * P * S);
-    L.v_mu = take(sizeof(float) * B * NP * P);
-    L.v_sum = take(2 * sizeof(float) * B * NP * P);
-    L.v_row_ticket = take(sizeof(unsigned) * B * NP);
+    L.v_mu = take(sizeof(float) * B * NP * VC);
+    L.v_sum = take(2 * sizeof(float) * B * NP * VC);
     L.v_table = take(sizeof(float) * B * NP * verify_table_width(c.K));
     L.v_rhat = take(sizeof(float) * B * NP * TL);
     L.r_best = take(sizeof(unsigned long long) * B * 3);
@@ -79,14 +78,6 @@ int sm_count() {
                                                    cudaSuccess || sms < 1)
         return 1;
     return sms;
-}
-
-// persistent grid: two CTAs per SM when the shared memory allows it, never
-// more CTAs than tiles (every CTA then owns at least one tile)
-int persistent_grid(int64_t tiles, size_t dyn_smem) {
-    const int per_sm = (dyn_smem + 16 * 1024) * 2 <= 227 * 1024 ? 2 : 1;
-    const int64_t g = (int64_t)sm_count() * per_sm;
-    return (int)(g < tiles ? g : tiles);
 }
 
 // largest number of segments any row is cut into by the tile split
@@ -106,10 +97,6 @@ bool rows_aligned(const void* p, int64_t row_stride, const rheo_config& c) {
     return ((uintptr_t)p % 16 == 0) && ((row_stride * elem_size(c)) % 16 == 0);
 }
 
-bool tma_ok(const void* p, int64_t row_stride, const rheo_config& c) {
-    const int es = elem_size(c);
-    return ((uintptr_t)p % 16 == 0) && ((row_stride * es) % 16 == 0) && (((int64_t)c.vocab * es) % 16 == 0);
-}
 
 Dims dims(const rheo_config& c) {
     Dims n;
@@ -190,7 +177,8 @@ extern "C" int rheo_expand(const rheo_config* cfg, int32_t d, const void* logits
     // needs no merge.  More rows: two CTAs per SM, rows cut where the even
     // split of the tiles falls.
     int grid;
-    if (rows <= sms) {
+    const bool whole = rows <= sms;
+    if (whole) {
         const int64_t P = std::max<int64_t>(1, std::min<int64_t>(tpr, sms / rows));
         grid = (int)(rows * P);
     } else {
@@ -200,7 +188,7 @@ extern "C" int rheo_expand(const rheo_config* cfg, int32_t d, const void* logits
     a.keys_bytes = expand_keys_bytes(segs, cfg->support);
     const size_t smem = expand_smem_bytes(segs, cfg->support);
     if (smem + 8 * 1024 > 227 * 1024) return RHEO_EINVAL;
-    return launch_expand(a, cfg->dtype, rows_aligned(logits, row_stride, *cfg), grid, smem, (cudaStream_t)stream) ==
+    return launch_expand(a, cfg->dtype, rows_aligned(logits, row_stride, *cfg), whole, grid, smem, (cudaStream_t)stream) ==
                    cudaSuccess
                ? RHEO_OK
                : RHEO_ELAUNCH;
@@ -245,18 +233,17 @@ extern "C" int rheo_verify(const rheo_config* cfg, const void* logits, int64_t r
     a.status = at<unsigned>(ws, L.status);
     a.seg_mu = at<float>(ws, L.v_mu);
     a.seg_sum = at<float>(ws, L.v_sum);
-    a.row_ticket = at<unsigned>(ws, L.v_row_ticket);
     a.table = at<float>(ws, L.v_table);
     a.rhat_tail = at<float>(ws, L.v_rhat);
     a.res_best = at<unsigned long long>(ws, L.r_best);
     a.res_ticket = at<unsigned>(ws, L.r_ticket);
     const int64_t NP = cfg->budget + 1;
-    const size_t stage = (size_t)NP * (verify_table_width(cfg->K) * 4 + 5 * 4);
-    a.table_smem_bytes = stage <= 160 * 1024 ? stage : 0;
-    const int tpr = tiles_per_row(*cfg);
-    const int grid = persistent_grid((int64_t)cfg->batch * NP * tpr, verify_stream_smem_bytes());
-    return launch_verify(a, cfg->dtype, tma_ok(logits, row_stride, *cfg), grid, verify_stream_smem_bytes(),
-                         (cudaStream_t)stream) == cudaSuccess
+    a.n.chunks = verify_chunks_per_row(cfg->dtype == RHEO_BF16 ? 1 : 0, cfg->vocab);
+    const int64_t chunks = (int64_t)cfg->batch * NP * a.n.chunks;
+    const int grid = verify_stream_grid(sm_count(), chunks);
+    a.units = verify_stream_units(grid, chunks);
+    return launch_verify(a, cfg->dtype, rows_aligned(logits, row_stride, *cfg), grid, (cudaStream_t)stream) ==
+                   cudaSuccess
                ? RHEO_OK
                : RHEO_ELAUNCH;
 }

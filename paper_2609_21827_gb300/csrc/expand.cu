@@ -31,8 +31,11 @@ namespace {
 
 constexpr int kRegion = 256;   // candidate keys per warp
 constexpr int kVPT = 4;        // 16-byte vectors per thread per tile
-constexpr int kBins = 4096;    // histogram of the top 12 key bits
-constexpr int kBinShift = 52;  // key >> kBinShift is the bin
+// two-level histogram of candidate keys: 256 coarse bins (top 8 key bits, two
+// octaves of value each) over 16384 fine bins (top 14 bits, 1/32 octave)
+constexpr int kCoarseBins = 256, kCoarseShift = 56;
+constexpr int kFineBins = 16384, kFineShift = 50;
+constexpr int kFinePerCoarse = kFineBins / kCoarseBins;
 
 struct E2Smem {
     unsigned long long sorted[kMaxSupport];
@@ -47,7 +50,7 @@ struct E2Smem {
 };
 
 struct HistSel {
-    int bin, above, tie_n;
+    int bin, cbin, above, tie_n;
 };
 
 __device__ __forceinline__ unsigned long long make_key(uint32_t k32, int64_t id) {
@@ -58,7 +61,7 @@ __device__ __forceinline__ unsigned long long make_key(uint32_t k32, int64_t id)
 // bound of the segment's S-th key.  cnt > S on entry.  The histogram loses the
 // keys that go.
 __device__ __noinline__ unsigned long long warp_cut_region(unsigned long long* region, int& cnt, int S,
-                                                           unsigned* vh) {
+                                                           unsigned* fine, unsigned* coarse) {
     const int lane = threadIdx.x & 31;
     unsigned long long x[kRegion / 32];
 #pragma unroll
@@ -72,7 +75,10 @@ __device__ __noinline__ unsigned long long warp_cut_region(unsigned long long* r
 #pragma unroll
     for (int i = 0; i < kRegion / 32; ++i) {
         const bool keep = x[i] != 0ull && x[i] >= thr;
-        if (x[i] != 0ull && !keep) atomicSub(&vh[(unsigned)(x[i] >> kBinShift)], 1u);
+        if (x[i] != 0ull && !keep) {
+            atomicSub(&fine[(unsigned)(x[i] >> kFineShift)], 1u);
+            atomicSub(&coarse[(unsigned)(x[i] >> kCoarseShift)], 1u);
+        }
         const unsigned bal = __ballot_sync(0xFFFFFFFFu, keep);
         if (keep) region[w + __popc(bal & ((1u << lane) - 1u))] = x[i];
         w += __popc(bal);
@@ -118,75 +124,156 @@ __device__ __forceinline__ void gather_at_least(Get get, int n, unsigned long lo
     }
 }
 
-// The k best of the distinct nonzero keys get(i), i < n, in descending order
-// into sorted[0, k); returns how many there are (min(k, number of keys)).
-// vh holds the keys' bin counts on entry; the bins that take part are left at
-// zero.  A scan of the histogram from the top gives every bin its offset in a
-// bin-ordered list; the keys of the bins down to the one holding the k-th key
-// are scattered there (tmp, tmp_cap entries) and each one is ranked among the
-// keys of its own bin only.  When that list would not fit (a huge tie class),
-// the k-th key is found by block_kth_key and the k keys are ranked directly.
-template <class Get>
-__device__ int hist_top_sorted(Get get, int n, int k, unsigned* vh, int* off, unsigned long long* tmp, int tmp_cap,
-                               unsigned long long* sorted, HistSel& hs, Red& red, int& par, unsigned* hist256,
-                               SelScratch& ss) {
-    constexpr int kPer = kBins / kThreads;
-    const int tid = threadIdx.x;
-    const int hi = kBins - 1 - tid * kPer;  // this thread's bins, from the top: hi, hi-1, ...
-    unsigned c[kPer];
-    int tot = 0;
+// One warp: the fine bin holding the k-th largest key counted by the two-level
+// histogram (coarse scan from the top, then the 64 fine bins of that coarse
+// bin).  bin = -1 when fewer than k keys are counted; above = keys in higher
+// fine bins.  Counts may change meanwhile (other warps insert or cut): a fine
+// level that lags its coarse level yields the coarse bin's lowest fine bin.
+__device__ __forceinline__ void warp_hist_find(const unsigned* coarse, const unsigned* fine, int k, int& bin,
+                                               int& above) {
+    const int lane = threadIdx.x & 31;
+    int acc = 0;
+    bin = -1;
+    above = 0;
+    for (int c0 = kCoarseBins - 1; c0 >= 0; c0 -= 32) {
+        const int v = (int)*reinterpret_cast<const volatile unsigned*>(&coarse[c0 - lane]);
+        int incl = v;
 #pragma unroll
-    for (int q = 0; q < kPer; ++q) {
-        c[q] = vh[hi - q];
-        tot += (int)c[q];
-    }
-    int total;
-    const int before = red_scan(tot, total, red, par);
-    const int kk = k < total ? k : total;
-    if (kk <= 0) return 0;
-    {
-        int acc = before;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        const int tot = __shfl_sync(0xFFFFFFFFu, incl, 31);
+        if (acc + tot < k) {
+            acc += tot;
+            continue;
+        }
+        const int L = __ffs(__ballot_sync(0xFFFFFFFFu, acc + incl >= k)) - 1;
+        const int cb = c0 - L;
+        int acc2 = acc + __shfl_sync(0xFFFFFFFFu, incl - v, L);
+        for (int f0 = cb * kFinePerCoarse + kFinePerCoarse - 1; f0 >= cb * kFinePerCoarse; f0 -= 32) {
+            const int w = (int)*reinterpret_cast<const volatile unsigned*>(&fine[f0 - lane]);
+            int inc2 = w;
 #pragma unroll
-        for (int q = 0; q < kPer; ++q) {
-            off[hi - q] = acc;
-            if (acc < kk && acc + (int)c[q] >= kk) {
-                hs.bin = hi - q;
-                hs.above = acc + (int)c[q];  // keys in the bins down to and with this one
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xFFFFFFFFu, inc2, o);
+                if (lane >= o) inc2 += y;
             }
-            acc += (int)c[q];
+            const int t2 = __shfl_sync(0xFFFFFFFFu, inc2, 31);
+            if (acc2 + t2 >= k) {
+                const int L2 = __ffs(__ballot_sync(0xFFFFFFFFu, acc2 + inc2 >= k)) - 1;
+                bin = f0 - L2;
+                above = acc2 + __shfl_sync(0xFFFFFFFFu, inc2 - w, L2);
+                return;
+            }
+            acc2 += t2;
+        }
+        bin = cb * kFinePerCoarse;
+        above = acc2;
+        return;
+    }
+}
+
+// Boundary of the k best keys counted by the two-level histogram: hs.bin = the
+// fine bin holding the k-th key (-1 when fewer than k keys are counted) and
+// hs.tie_n = 0.  Thread t scans coarse bin 255 - t (a block scan from the top),
+// then one warp scans the 64 fine bins of the coarse bin found.
+__device__ void hist_boundary(const unsigned* coarse, const unsigned* fine, int k, HistSel& hs, Red& red, int& par) {
+    static_assert(kCoarseBins == kThreads, "one coarse bin per thread");
+    const int tid = threadIdx.x, lane = tid & 31;
+    const int cb = kCoarseBins - 1 - tid;
+    const int c = (int)coarse[cb];
+    int total;
+    const int before = red_scan(c, total, red, par);
+    if (tid == 0) {
+        hs.bin = -1;
+        hs.tie_n = 0;
+    }
+    if (total >= k && before < k && before + c >= k) {
+        hs.cbin = cb;
+        hs.above = before;
+    }
+    __syncthreads();
+    if (total >= k && tid < 32) {
+        const int cbin = hs.cbin;
+        int acc = hs.above;
+        for (int f0 = cbin * kFinePerCoarse + kFinePerCoarse - 1; f0 >= cbin * kFinePerCoarse; f0 -= 32) {
+            const int w = (int)fine[f0 - lane];
+            int inc = w;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+                if (lane >= o) inc += y;
+            }
+            const int t2 = __shfl_sync(0xFFFFFFFFu, inc, 31);
+            if (acc + t2 >= k) {
+                const int L2 = __ffs(__ballot_sync(0xFFFFFFFFu, acc + inc >= k)) - 1;
+                if (lane == 0) hs.bin = f0 - L2;
+                break;
+            }
+            acc += t2;
         }
     }
     __syncthreads();
-    const int bstar = hs.bin, nsel = hs.above;
-    if (nsel <= tmp_cap) {
-        for (int i = tid; i < n; i += kThreads) {
-            const unsigned long long x = get(i);
-            const int b = (int)(x >> kBinShift);
-            if (x != 0ull && b >= bstar) tmp[off[b] + (int)atomicSub(&vh[b], 1u) - 1] = x;
-        }
-        __syncthreads();
-        for (int p = tid; p < nsel; p += kThreads) {
-            const unsigned long long x = tmp[p];
-            const int b = (int)(x >> kBinShift);
-            const int s0 = off[b], e = (b == bstar) ? nsel : off[b - 1];
-            int rank = 0;
-            for (int q = s0; q < e; ++q) rank += tmp[q] > x;
-            if (s0 + rank < kk) sorted[s0 + rank] = x;
-        }
-        __syncthreads();
-        return kk;
+}
+
+// Append the keys x with fine bin >= bin among xs[0, cnt) (this warp's keys) to
+// tmp at positions from hs.tie_n, one shared atomic per 32 keys.
+__device__ __forceinline__ void warp_gather_from(const unsigned long long* xs, int cnt, int bin,
+                                                 unsigned long long* tmp, int cap, HistSel& hs) {
+    const int lane = threadIdx.x & 31;
+    for (int j0 = 0; j0 < cnt; j0 += 32) {
+        const unsigned long long x = (j0 + lane < cnt) ? xs[j0 + lane] : 0ull;
+        const bool take = x != 0ull && (int)(x >> kFineShift) >= bin;
+        const unsigned bal = __ballot_sync(0xFFFFFFFFu, take);
+        int base = 0;
+        if (lane == 0 && bal) base = atomicAdd(&hs.tie_n, __popc(bal));
+        base = __shfl_sync(0xFFFFFFFFu, base, 0);
+        const int pos = base + __popc(bal & ((1u << lane) - 1u));
+        if (take && pos < cap) tmp[pos] = x;
     }
-    // a tie class too large for the list
-    const unsigned long long thr = block_kth_key(get, n, kk, hist256, ss);
-    if (tid == 0) hs.tie_n = 0;
+}
+
+// Block-wide: append the keys with fine bin >= bin among get(i), i < n.
+template <class Get>
+__device__ __forceinline__ void block_gather_bin(Get get, int n, int bin, unsigned long long* tmp, int cap,
+                                                 HistSel& hs) {
+    const int lane = threadIdx.x & 31;
+    for (int i0 = 0; i0 < n; i0 += kThreads) {
+        const int i = i0 + (int)threadIdx.x;
+        const unsigned long long x = i < n ? get(i) : 0ull;
+        const bool take = x != 0ull && (int)(x >> kFineShift) >= bin;
+        const unsigned bal = __ballot_sync(0xFFFFFFFFu, take);
+        int base = 0;
+        if (lane == 0 && bal) base = atomicAdd(&hs.tie_n, __popc(bal));
+        base = __shfl_sync(0xFFFFFFFFu, base, 0);
+        const int pos = base + __popc(bal & ((1u << lane) - 1u));
+        if (take && pos < cap) tmp[pos] = x;
+    }
+}
+
+// The gathered keys tmp[0, hs.tie_n) ranked: the k best in descending order into
+// sorted[0, k); returns how many (min(k, gathered)).  Two threads rank each key.
+__device__ int rank_gathered(const unsigned long long* tmp, int k, unsigned long long* sorted, HistSel& hs) {
     __syncthreads();
-    gather_at_least(get, n, thr, tmp, kk, &hs.tie_n);
-    __syncthreads();
-    for (int p = tid; p < kk; p += kThreads) {
-        const unsigned long long x = tmp[p];
+    const int nsel = hs.tie_n;
+    const int kk = nsel < k ? nsel : k;
+    for (int p0 = 0; p0 < nsel; p0 += kThreads / 2) {
+        const int p = p0 + ((int)threadIdx.x >> 1), h = threadIdx.x & 1;
+        const unsigned long long x = p < nsel ? tmp[p] : 0ull;
         int rank = 0;
-        for (int q = 0; q < kk; ++q) rank += tmp[q] > x;
-        if (rank < kk) sorted[rank] = x;
+        if (p < nsel) {
+            int r0 = 0, r1 = 0;
+            int q = h;
+            for (; q + 2 < nsel; q += 4) {
+                r0 += tmp[q] > x;
+                r1 += tmp[q + 2] > x;
+            }
+            for (; q < nsel; q += 2) r0 += tmp[q] > x;
+            rank = r0 + r1;
+        }
+        rank += __shfl_xor_sync(0xFFFFFFFFu, rank, 1);
+        if (p < nsel && h == 0 && rank < kk) sorted[rank] = x;
     }
     __syncthreads();
     return kk;
@@ -197,15 +284,15 @@ __device__ int hist_top_sorted(Get get, int n, int k, unsigned* vh, int* off, un
 // keys below theta dropped, the region cut to its S best whenever it fills.
 template <int DT>
 __device__ __noinline__ void insert_rounds(unsigned long long* region, int& cnt, uint32_t pend, const uint4* wspill,
-                                           int e0, unsigned long long& theta, int S, unsigned* vh,
-                                           unsigned long long* s_theta) {
+                                           int e0, unsigned long long& theta, int S, unsigned* fine,
+                                           unsigned* coarse, unsigned long long* s_theta) {
     using E = Elem<DT>;
     constexpr int VEC = E::VEC;
     const int lane = threadIdx.x & 31, tid = threadIdx.x;
     const uint32_t* wv0 = reinterpret_cast<const uint32_t*>(wspill);
     while (__any_sync(0xFFFFFFFFu, pend != 0u)) {
         if (cnt > kRegion - 32) {
-            const unsigned long long thr = warp_cut_region(region, cnt, S, vh);
+            const unsigned long long thr = warp_cut_region(region, cnt, S, fine, coarse);
             if (lane == 0) atomicMax(s_theta, thr);
             theta = thr > theta ? thr : theta;
         }
@@ -222,7 +309,8 @@ __device__ __noinline__ void insert_rounds(unsigned long long* region, int& cnt,
         const unsigned bal = __ballot_sync(0xFFFFFFFFu, x != 0ull);
         if (x) {
             region[cnt + __popc(bal & ((1u << lane) - 1u))] = x;
-            atomicAdd(&vh[(unsigned)(x >> kBinShift)], 1u);
+            atomicAdd(&fine[(unsigned)(x >> kFineShift)], 1u);
+            atomicAdd(&coarse[(unsigned)(x >> kCoarseShift)], 1u);
         }
         cnt += __popc(bal);
     }
@@ -230,14 +318,13 @@ __device__ __noinline__ void insert_rounds(unsigned long long* region, int& cnt,
 
 }  // namespace
 
-template <int DT, bool ALIGNED>
-__global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a) {
+template <int DT, bool ALIGNED, int NS>
+__global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const ExpandArgs a) {
     using E = Elem<DT>;
     using W = Vec<DT>;
     constexpr int VEC = E::VEC;
     constexpr int TE = kTileBytes / E::SIZE;  // elements per tile
     static_assert(TE == kVPT * VEC * kThreads, "tile layout");
-    static_assert(kBins % kThreads == 0, "histogram split");
     constexpr float kLog2e = 1.4426950408889634f;
     extern __shared__ __align__(128) unsigned char dsm[];
     // per-warp candidate regions; after a segment's selection the same space
@@ -245,8 +332,8 @@ __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a)
     unsigned long long* keys = reinterpret_cast<unsigned long long*>(dsm);
     // per-warp copy of the lanes' vectors of a tile that has candidates
     uint4* spill = reinterpret_cast<uint4*>(dsm + a.keys_bytes);
-    unsigned* vh = reinterpret_cast<unsigned*>(dsm + a.keys_bytes + sizeof(uint4) * kWarps * 32 * kVPT);
-    int* off = reinterpret_cast<int*>(vh + kBins);  // bin offsets of the top-S sort
+    unsigned* fine = reinterpret_cast<unsigned*>(dsm + a.keys_bytes + sizeof(uint4) * kWarps * 32 * kVPT);
+    unsigned* coarse = fine + kFineBins;
     // the spill area doubles as the bin-ordered list of the top-S sort
     unsigned long long* tmpk = reinterpret_cast<unsigned long long*>(spill);
     constexpr int kTmpCap = kWarps * 32 * kVPT * (int)sizeof(uint4) / (int)sizeof(unsigned long long);
@@ -278,40 +365,21 @@ __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a)
     unsigned long long theta = 0ull;
     int cnt = 0, seg_tiles = 0;
     int64_t seg_valid = 0;
-    int64_t r = t0 / tpr;
-    int tt = (int)(t0 % tpr);
-    uint4 nxt[kVPT];
-    if (t0 < t1) load_tile<DT, ALIGNED>(nxt, a.logits + r * a.row_stride_bytes, tt * TE, V);
-    for (int64_t t = t0; t < t1; ++t, ++tt) {
-        if (tt == tpr) {
-            tt = 0;
-            ++r;
-        }
-        const bool seg_first = (t == t0) || (tt == 0);
-        const bool seg_last = (t == t1 - 1) || (tt == tpr - 1);
-        const int e0 = tt * TE;
-        const int ne = min(TE, V - e0);
-        uint4 v[kVPT];
-#pragma unroll
-        for (int j = 0; j < kVPT; ++j) v[j] = nxt[j];
-        if (t + 1 < t1) {  // the next tile is in flight while this one is worked on
-            const bool wrap = (tt + 1 == tpr);
-            load_tile<DT, ALIGNED>(nxt, a.logits + (r + (wrap ? 1 : 0)) * a.row_stride_bytes, wrap ? 0 : e0 + TE, V);
-        }
-        float vm[kVPT];
+
+    auto seg_begin = [&]() {
+        mu = -INFINITY;
+        sum = 0.0f;
+        seg_valid = 0;
+        cnt = 0;
+        for (int i = tid; i < (kFineBins + kCoarseBins) / 4; i += kThreads)
+            reinterpret_cast<uint4*>(fine)[i] = make_uint4(0u, 0u, 0u, 0u);
+    };
+    // running partition sum at T = 1 (online max); mu is also the running
+    // maximum of this thread's elements
+    auto tile_sum = [&](const uint4 (&v)[kVPT], float (&vm)[kVPT]) {
 #pragma unroll
         for (int j = 0; j < kVPT; ++j) vm[j] = W::vmax(v[j]);
         const float tmax = fmaxf(fmaxf(vm[0], vm[1]), fmaxf(vm[2], vm[3]));
-
-        if (seg_first) {
-            mu = -INFINITY;
-            sum = 0.0f;
-            seg_valid = 0;
-            cnt = 0;
-            for (int i = tid; i < kBins; i += kThreads) vh[i] = 0u;
-        }
-        // running partition sum at T = 1 (online max); mu is also the running
-        // maximum of this thread's elements
         if (tmax > mu) {
             if (mu != -INFINITY) sum *= fast_exp2((mu - tmax) * kLog2e);
             mu = tmax;
@@ -321,11 +389,17 @@ __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a)
             sum += (W::vexp(v[0], kLog2e, mc) + W::vexp(v[1], kLog2e, mc)) +
                    (W::vexp(v[2], kLog2e, mc) + W::vexp(v[3], kLog2e, mc));
         }
-        // on the segment's tiles 1, 2, 4, 8, ... this warp's bound: the kb-th
-        // largest running maximum of its lanes (lanes with no element count as
-        // absent); kb lanes hold an element at or above it
+    };
+    // The bound theta.  On the first step of a segment: every warp's kb-th
+    // largest running maximum of its lanes (lanes with no element count as
+    // absent) -- kb lanes hold an element at or above it, so at least S elements
+    // reach the smallest of those bounds; the block synchronises on it.  On every
+    // later step one warp in turn finds, in the histogram of the candidates so
+    // far, the fine bin of the S-th key: at least S elements lie at or above
+    // that bin's lower edge, which becomes the shared bound.
+    auto refresh = [&](bool seg_first) {
         seg_tiles = seg_first ? 1 : seg_tiles + 1;
-        if ((seg_tiles & (seg_tiles - 1)) == 0) {
+        if (seg_first) {
             const uint32_t lk = (mu > -INFINITY) ? E::key_of_value(mu) : 0u;
             int rank = 0;
 #pragma unroll
@@ -335,82 +409,79 @@ __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a)
             }
             const unsigned who = __ballot_sync(0xFFFFFFFFu, rank == kb - 1);
             const uint32_t wb = __shfl_sync(0xFFFFFFFFu, lk, __ffs(who) - 1);
-            if (lane == 0) s_wb[warp] = wb;  // bounds only grow within a segment
+            if (lane == 0) s_wb[warp] = wb;
+            __syncthreads();
+            uint32_t b = s_wb[0];
+#pragma unroll
+            for (int w = 1; w < kWarps; ++w) b = min(b, s_wb[w]);
+            theta = (unsigned long long)b << 32;
+        } else if (seg_tiles % kWarps == warp) {
+            int bin, above;
+            warp_hist_find(coarse, fine, S, bin, above);
+            if (bin >= 0) {
+                const unsigned long long hb = (unsigned long long)bin << kFineShift;
+                if (lane == 0) atomicMax(&s_theta, hb);
+                theta = hb > theta ? hb : theta;
+            }
         }
-        // every warp has kb elements at or above its bound, so at least S elements
-        // reach the smallest bound (read again after a refresh, and on the tile
-        // after it, when the other warps have refreshed too)
-        if (seg_first) __syncthreads();
-        if (seg_tiles <= 2 || ((seg_tiles - 1) & (seg_tiles - 2)) == 0 || (seg_tiles & (seg_tiles - 1)) == 0) {
-            uint32_t b = *reinterpret_cast<volatile uint32_t*>(&s_wb[0]);
+        const unsigned long long ts = *reinterpret_cast<volatile unsigned long long*>(&s_theta);
+        theta = ts > theta ? ts : theta;
+    };
+    // candidates of one tile: elements whose value reaches theta's (a superset
+    // of the keys >= theta; the final selection is exact).  Every lane writes its
+    // own at offsets from a warp scan.
+    auto tile_candidates = [&](const uint4 (&v)[kVPT], const float (&vm)[kVPT], int e0, int ne) {
+        const float thv = E::threshold_value((uint32_t)(theta >> 32));
+        uint32_t pend = 0u;
 #pragma unroll
-            for (int w = 1; w < kWarps; ++w) b = min(b, *reinterpret_cast<volatile uint32_t*>(&s_wb[w]));
-            const unsigned long long tb = (unsigned long long)b << 32;
-            theta = seg_first ? tb : (tb > theta ? tb : theta);
-        }
-        {
-            const unsigned long long ts = *reinterpret_cast<volatile unsigned long long*>(&s_theta);
-            theta = ts > theta ? ts : theta;
-        }
-        seg_valid += ne;
-
-
-        // candidates: elements whose value reaches theta's (a superset of the keys
-        // >= theta; the final selection is exact).  Every lane writes its own at
-        // offsets from a warp scan.
-        auto screen = [&](float thv) -> uint32_t {
-            uint32_t pm = 0u;
+        for (int j = 0; j < kVPT; ++j)
+            if (vm[j] >= thv) {
+                if (ne == TE) {
 #pragma unroll
-            for (int j = 0; j < kVPT; ++j)
-                if (vm[j] >= thv) {
-                    if (ne == TE) {
+                    for (int i = 0; i < VEC; ++i)
+                        pend |= (E::value(E::raw(v[j], i)) >= thv) ? (1u << (j * VEC + i)) : 0u;
+                } else {
 #pragma unroll
-                        for (int i = 0; i < VEC; ++i)
-                            pm |= (E::value(E::raw(v[j], i)) >= thv) ? (1u << (j * VEC + i)) : 0u;
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < VEC; ++i) {
-                            const bool in = (j * kThreads + tid) * VEC + i < ne;
-                            pm |= (in && E::value(E::raw(v[j], i)) >= thv) ? (1u << (j * VEC + i)) : 0u;
-                        }
+                    for (int i = 0; i < VEC; ++i) {
+                        const bool in = (j * kThreads + tid) * VEC + i < ne;
+                        pend |= (in && E::value(E::raw(v[j], i)) >= thv) ? (1u << (j * VEC + i)) : 0u;
                     }
                 }
-            return pm;
-        };
-        uint32_t pend = screen(E::threshold_value((uint32_t)(theta >> 32)));
-        if (__any_sync(0xFFFFFFFFu, pend != 0u)) {
-#pragma unroll
-            for (int j = 0; j < kVPT; ++j) wspill[j * 32 + lane] = v[j];
-            const int c = __popc(pend);
-            int incl = c;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-                if (lane >= o) incl += y;
             }
-            const int total = __shfl_sync(0xFFFFFFFFu, incl, 31);
-            if (cnt + total <= kRegion) {
-                const uint32_t* wv0 = reinterpret_cast<const uint32_t*>(wspill);
-                int pos = cnt + incl - c;
-                for (uint32_t mm = pend; mm; mm &= mm - 1u) {
-                    const int q = __ffs(mm) - 1;
-                    const int j = q / VEC, i = q % VEC;
-                    const uint32_t* wv = wv0 + (j * 32 + lane) * 4;
-                    const uint32_t raw = (DT == 0) ? wv[i] : ((wv[i >> 1] >> ((i & 1) * 16)) & 0xFFFFu);
-                    const unsigned long long x = make_key(E::key(raw), (int64_t)e0 + (j * kThreads + tid) * VEC + i);
-                    region[pos++] = x;
-                    atomicAdd(&vh[(unsigned)(x >> kBinShift)], 1u);
-                }
-                cnt += total;
-            } else {
-                // the region would overflow: one candidate per lane and round,
-                // keys below theta dropped, the region cut whenever it fills
-                insert_rounds<DT>(region, cnt, pend, wspill, e0, theta, S, vh, &s_theta);
-            }
-            __syncwarp();
+        if (!__any_sync(0xFFFFFFFFu, pend != 0u)) return;
+#pragma unroll
+        for (int j = 0; j < kVPT; ++j) wspill[j * 32 + lane] = v[j];
+        const int c = __popc(pend);
+        int incl = c;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+            if (lane >= o) incl += y;
         }
-        if (!seg_last) continue;
-
+        const int total = __shfl_sync(0xFFFFFFFFu, incl, 31);
+        if (cnt + total <= kRegion) {
+            const uint32_t* wv0 = reinterpret_cast<const uint32_t*>(wspill);
+            int pos = cnt + incl - c;
+            for (uint32_t mm = pend; mm; mm &= mm - 1u) {
+                const int q = __ffs(mm) - 1;
+                const int j = q / VEC, i = q % VEC;
+                const uint32_t* wv = wv0 + (j * 32 + lane) * 4;
+                const uint32_t raw = (DT == 0) ? wv[i] : ((wv[i >> 1] >> ((i & 1) * 16)) & 0xFFFFu);
+                const unsigned long long x = make_key(E::key(raw), (int64_t)e0 + (j * kThreads + tid) * VEC + i);
+                region[pos++] = x;
+                atomicAdd(&fine[(unsigned)(x >> kFineShift)], 1u);
+                atomicAdd(&coarse[(unsigned)(x >> kCoarseShift)], 1u);
+            }
+            cnt += total;
+        } else {
+            // the region would overflow: one candidate per lane and round, keys
+            // below theta dropped, the region cut whenever it fills
+            insert_rounds<DT>(region, cnt, pend, wspill, e0, theta, S, fine, coarse, &s_theta);
+        }
+        __syncwarp();
+    };
+    // end of the segment of row r that this CTA holds
+    auto segment_end = [&](int64_t r) {
         // ---- end of segment: exact top-S keys ------------------------------------
         if (lane == 0) s_rcount[warp] = cnt;
         float Ms;
@@ -420,8 +491,20 @@ __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a)
         auto rkey = [&](int i) -> unsigned long long {
             return (i % kRegion) < s_rcount[i / kRegion] ? keys[i] : 0ull;
         };
-        const int written = hist_top_sorted(rkey, kWarps * kRegion, target, vh, off, tmpk, kTmpCap, e2.sorted, hs,
-                                            red, par, s_hist, s_sel);
+        // the k best: all keys at or above the fine bin of the k-th, ranked
+        hist_boundary(coarse, fine, target, hs, red, par);
+        warp_gather_from(region, cnt, hs.bin < 0 ? 0 : hs.bin, tmpk, kTmpCap, hs);
+        __syncthreads();
+        int written;
+        if (hs.tie_n <= kTmpCap) {
+            written = rank_gathered(tmpk, target, e2.sorted, hs);
+        } else {  // a tie class too large for the list
+            const unsigned long long thr = block_kth_key(rkey, kWarps * kRegion, target, s_hist, s_sel);
+            if (tid == 0) hs.tie_n = 0;
+            __syncthreads();
+            gather_at_least(rkey, kWarps * kRegion, thr, tmpk, target, &hs.tie_n);
+            written = rank_gathered(tmpk, target, e2.sorted, hs);
+        }
         const int first_owner = sp.owner(r * tpr);
         const int seg = (int)blockIdx.x - first_owner;
         const int nseg = sp.owner(r * tpr + tpr - 1) - first_owner + 1;
@@ -445,21 +528,37 @@ __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a)
                 a.seg_sum[2 * ((int64_t)r * tpr + seg)] = Ss.hi;
                 a.seg_sum[2 * ((int64_t)r * tpr + seg) + 1] = Ss.lo;
             }
-            if (!arrive_last(a.row_ticket + r, (unsigned)nseg, bs)) continue;
+            if (!arrive_last(a.row_ticket + r, (unsigned)nseg, bs)) return;
 
             // ---- last segment of row r: merge the segments' lists and sums ---------
             const int nkeys = nseg * S;
             const unsigned long long* rk = a.seg_keys + (int64_t)r * tpr * S;
-            for (int i = tid; i < kBins; i += kThreads) vh[i] = 0u;
+            for (int i = tid; i < (kFineBins + kCoarseBins) / 4; i += kThreads)
+                reinterpret_cast<uint4*>(fine)[i] = make_uint4(0u, 0u, 0u, 0u);
             __syncthreads();
             for (int i = tid; i < nkeys; i += kThreads) {
                 const unsigned long long x = __ldcg(rk + i);
                 keys[i] = x;
-                if (x) atomicAdd(&vh[(unsigned)(x >> kBinShift)], 1u);
+                if (x) {
+                    atomicAdd(&fine[(unsigned)(x >> kFineShift)], 1u);
+                    atomicAdd(&coarse[(unsigned)(x >> kCoarseShift)], 1u);
+                }
             }
             __syncthreads();
-            const int got = hist_top_sorted([&](int i) { return keys[i]; }, nkeys, S, vh, off, tmpk, kTmpCap,
-                                            e2.sorted, hs, red, par, s_hist, s_sel);
+            auto mkey = [&](int i) { return keys[i]; };
+            hist_boundary(coarse, fine, S, hs, red, par);
+            block_gather_bin(mkey, nkeys, hs.bin < 0 ? 0 : hs.bin, tmpk, kTmpCap, hs);
+            __syncthreads();
+            int got;
+            if (hs.tie_n <= kTmpCap) {
+                got = rank_gathered(tmpk, S, e2.sorted, hs);
+            } else {
+                const unsigned long long thr = block_kth_key(mkey, nkeys, S, s_hist, s_sel);
+                if (tid == 0) hs.tie_n = 0;
+                __syncthreads();
+                gather_at_least(mkey, nkeys, thr, tmpk, S, &hs.tie_n);
+                got = rank_gathered(tmpk, S, e2.sorted, hs);
+            }
             if (tid < 32) {
                 float mx = -INFINITY;
                 for (int c = tid; c < nseg; c += 32) mx = fmaxf(mx, __ldcg(a.seg_mu + (int64_t)r * tpr + c));
@@ -582,8 +681,8 @@ __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a)
         if (tid == 0) a.tree.lse1[(int64_t)b * n.E + eidx] = lse1;
 
         // ---- last row of the request: the K best depth-d nodes become the frontier ----
-        if (!arrive_last(a.req_ticket + b, (unsigned)a.F, bs)) continue;
-        if (a.d == n.D) continue;
+        if (!arrive_last(a.req_ticket + b, (unsigned)a.F, bs)) return;
+        if (a.d == n.D) return;
         {
             const int nn = a.F * (K + 1);
             const int64_t base = depth_base(K, a.d);
@@ -621,18 +720,88 @@ __global__ void __launch_bounds__(kThreads, 2) expand_kernel(const ExpandArgs a)
             }
             __syncthreads();
         }
+    };
+
+    if (NS == 1) {
+        // the CTA's tiles in order; segments end at row boundaries
+        int64_t r = t0 / tpr;
+        int tt = (int)(t0 % tpr);
+        uint4 nxt[kVPT];
+        if (t0 < t1) load_tile<DT, ALIGNED>(nxt, a.logits + r * a.row_stride_bytes, tt * TE, V);
+        for (int64_t t = t0; t < t1; ++t, ++tt) {
+            if (tt == tpr) {
+                tt = 0;
+                ++r;
+            }
+            const bool seg_first = (t == t0) || (tt == 0);
+            const bool seg_last = (t == t1 - 1) || (tt == tpr - 1);
+            const int e0 = tt * TE;
+            const int ne = min(TE, V - e0);
+            uint4 v[kVPT];
+#pragma unroll
+            for (int j = 0; j < kVPT; ++j) v[j] = nxt[j];
+            if (t + 1 < t1) {  // the next tile is in flight while this one is worked on
+                const bool wrap = (tt + 1 == tpr);
+                load_tile<DT, ALIGNED>(nxt, a.logits + (r + (wrap ? 1 : 0)) * a.row_stride_bytes, wrap ? 0 : e0 + TE, V);
+            }
+            if (seg_first) seg_begin();
+            float vm[kVPT];
+            tile_sum(v, vm);
+            refresh(seg_first);
+            seg_valid += ne;
+            tile_candidates(v, vm, e0, ne);
+            if (seg_last) segment_end(r);
+        }
+    } else {
+        // the CTA's tiles lie in one row: its two halves are streamed side by
+        // side, two tiles in flight per step
+        if (t0 >= t1) return;
+        const int64_t r = t0 / tpr;
+        const char* row = a.logits + r * a.row_stride_bytes;
+        const int ta = (int)(t0 % tpr);
+        const int len = (int)(t1 - t0), la = (len + 1) / 2, tb = ta + la, lb = len - la;
+        uint4 nxa[kVPT], nxb[kVPT];
+        load_tile<DT, ALIGNED>(nxa, row, ta * TE, V);
+        if (lb > 0) load_tile<DT, ALIGNED>(nxb, row, tb * TE, V);
+        seg_begin();
+        for (int i = 0; i < la; ++i) {
+            const bool hb = i < lb;
+            const int ea = (ta + i) * TE, eb = (tb + i) * TE;
+            const int na = min(TE, V - ea), nb = hb ? min(TE, V - eb) : 0;
+            uint4 va[kVPT], vb[kVPT];
+#pragma unroll
+            for (int j = 0; j < kVPT; ++j) {
+                va[j] = nxa[j];
+                vb[j] = nxb[j];
+            }
+            if (i + 1 < la) load_tile<DT, ALIGNED>(nxa, row, ea + TE, V);
+            if (i + 1 < lb) load_tile<DT, ALIGNED>(nxb, row, eb + TE, V);
+            float vma[kVPT], vmb[kVPT];
+            tile_sum(va, vma);
+            if (hb) tile_sum(vb, vmb);
+            refresh(i == 0);
+            seg_valid += na + nb;
+            tile_candidates(va, vma, ea, na);
+            if (hb) tile_candidates(vb, vmb, eb, nb);
+        }
+        segment_end(r);
     }
 }
 
-cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, int grid, size_t smem, cudaStream_t s) {
+cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, bool whole, int grid, size_t smem,
+                          cudaStream_t s) {
     auto go = [&](auto kern) {
         cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (err != cudaSuccess) return err;
         kern<<<grid, kThreads, smem, s>>>(a);
         return cudaGetLastError();
     };
-    if (dtype == 1) return aligned ? go(expand_kernel<1, true>) : go(expand_kernel<1, false>);
-    return aligned ? go(expand_kernel<0, true>) : go(expand_kernel<0, false>);
+    if (whole) {
+        if (dtype == 1) return aligned ? go(expand_kernel<1, true, 2>) : go(expand_kernel<1, false, 2>);
+        return aligned ? go(expand_kernel<0, true, 2>) : go(expand_kernel<0, false, 2>);
+    }
+    if (dtype == 1) return aligned ? go(expand_kernel<1, true, 1>) : go(expand_kernel<1, false, 1>);
+    return aligned ? go(expand_kernel<0, true, 1>) : go(expand_kernel<0, false, 1>);
 }
 
 size_t expand_keys_bytes(int max_segments, int support) {
@@ -642,7 +811,8 @@ size_t expand_keys_bytes(int max_segments, int support) {
 }
 
 size_t expand_smem_bytes(int max_segments, int support) {
-    return expand_keys_bytes(max_segments, support) + sizeof(uint4) * kWarps * 32 * kVPT + 2 * sizeof(unsigned) * kBins;
+    return expand_keys_bytes(max_segments, support) + sizeof(uint4) * kWarps * 32 * kVPT +
+           sizeof(unsigned) * (kFineBins + kCoarseBins);
 }
 
 int expand_tile_elems(int dtype) { return kTileBytes / (dtype == 1 ? 2 : 4); }

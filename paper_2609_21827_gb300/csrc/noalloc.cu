@@ -51,19 +51,17 @@ size_t up256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 // the verification part of the workspace layout, laid out in the static array
 struct StaticLayout {
-    size_t status, mu, sum, row_ticket, table, rhat, best, res_ticket, total, clear_end;
+    size_t status, mu, sum, table, rhat, best, res_ticket, total, clear_end;
 };
 
 StaticLayout static_layout(const rheo_config& c) {
     const int64_t B = c.batch, NP = c.budget + 1, TL = c.support - c.m;
-    const int te = verify_tile_elems(c.dtype == RHEO_BF16 ? 1 : 0);
-    const int64_t P = (c.vocab + te - 1) / te;
+    const int64_t P = verify_chunks_per_row(c.dtype == RHEO_BF16 ? 1 : 0, c.vocab);
     StaticLayout L{};
     size_t o = 0;
     auto take = [&](size_t bytes) { size_t at = o; o = up256(o + bytes); return at; };
     // everything that must start at zero first, so one memset clears it
     L.status = take(sizeof(unsigned));
-    L.row_ticket = take(sizeof(unsigned) * B * NP);
     L.best = take(sizeof(unsigned long long) * B * 3);
     L.res_ticket = take(sizeof(unsigned) * B);
     L.clear_end = o;
@@ -117,8 +115,7 @@ extern "C" int rheo_verify_static(const rheo_config* cfg, const void* logits, in
     a.n.N = cfg->budget;
     a.n.TL = cfg->support - cfg->m;
     a.n.GW = (cfg->K + 1) + a.n.TL;
-    const int te = verify_tile_elems(cfg->dtype == RHEO_BF16 ? 1 : 0);
-    a.n.chunks = (cfg->vocab + te - 1) / te;
+    a.n.chunks = verify_chunks_per_row(cfg->dtype == RHEO_BF16 ? 1 : 0, cfg->vocab);
     a.n.G1 = 1 + (int64_t)(cfg->K + 1) + (int64_t)(cfg->depth - 1) * cfg->K * (cfg->K + 1);
     a.n.E = 1 + (int64_t)(cfg->depth - 1) * cfg->K;
     a.n.eps = cfg->eps;
@@ -140,23 +137,18 @@ extern "C" int rheo_verify_static(const rheo_config* cfg, const void* logits, in
     a.status = reinterpret_cast<unsigned*>(base + L.status);
     a.seg_mu = reinterpret_cast<float*>(base + L.mu);
     a.seg_sum = reinterpret_cast<float*>(base + L.sum);
-    a.row_ticket = reinterpret_cast<unsigned*>(base + L.row_ticket);
     a.table = reinterpret_cast<float*>(base + L.table);
     a.rhat_tail = reinterpret_cast<float*>(base + L.rhat);
     a.res_best = reinterpret_cast<unsigned long long*>(base + L.best);
     a.res_ticket = reinterpret_cast<unsigned*>(base + L.res_ticket);
-    const size_t stage = (size_t)(cfg->budget + 1) * (verify_table_width(cfg->K) * 4 + 5 * 4);
-    a.table_smem_bytes = stage <= 160 * 1024 ? stage : 0;
-
     int sms = 1, dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
         return RHEO_ELAUNCH;
-    const int64_t tiles = (int64_t)cfg->batch * (cfg->budget + 1) * a.n.chunks;
-    const size_t smem = verify_stream_smem_bytes();
-    const int per_sm = (smem + 16 * 1024) * 2 <= 227 * 1024 ? 2 : 1;
-    const int grid = (int)(tiles < (int64_t)sms * per_sm ? tiles : (int64_t)sms * per_sm);
-    const bool tma = ((uintptr_t)logits % 16 == 0) && ((row_stride * es) % 16 == 0) && (((int64_t)cfg->vocab * es) % 16 == 0);
-    if (launch_verify(a, cfg->dtype, tma, grid, smem, s) != cudaSuccess) return RHEO_ELAUNCH;
+    const int64_t chunks = (int64_t)cfg->batch * (cfg->budget + 1) * a.n.chunks;
+    const int grid = verify_stream_grid(sms, chunks);
+    a.units = verify_stream_units(grid, chunks);
+    const bool aligned = ((uintptr_t)logits % 16 == 0) && ((row_stride * es) % 16 == 0);
+    if (launch_verify(a, cfg->dtype, aligned, grid, s) != cudaSuccess) return RHEO_ELAUNCH;
     if (status && cudaMemcpyAsync(status, base + L.status, sizeof(int32_t), cudaMemcpyDeviceToDevice, s) != cudaSuccess)
         return RHEO_ELAUNCH;
     return RHEO_OK;

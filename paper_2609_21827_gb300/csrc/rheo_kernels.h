@@ -64,7 +64,8 @@ struct PruneArgs {
 };
 
 struct VerifyArgs {
-    Dims n;
+    Dims n;                         // n.chunks: 2 KB chunks per target row
+    int units;                      // warps of the stream launch with work (one contiguous run of chunks each)
     const char* logits;
     int64_t row_stride_bytes;
     const float* T;
@@ -78,27 +79,28 @@ struct VerifyArgs {
     int32_t* bonus_token;
     float* row_lse;                 // may be null
     unsigned* status;
-    float* seg_mu;                  // [B*(N+1)*tiles_per_row]
-    float* seg_sum;                 // [B*(N+1)*tiles_per_row*2] float-float partition sums
-    unsigned* row_ticket;           // [B*(N+1)]
+    float* seg_mu;                  // [B*(N+1)*chunks]
+    float* seg_sum;                 // [B*(N+1)*chunks*2] float-float partition sums
     float* table;                   // [B*(N+1)*table_width(K)] decision tables
     float* rhat_tail;               // [B*(N+1)*TL]
     unsigned long long* res_best;   // [B*3]
     unsigned* res_ticket;           // [B]
-    size_t table_smem_bytes;        // dynamic shared memory of the residual kernel
 };
 
 // Host launchers, defined next to their kernels.  dtype: 0 fp32, 1 bf16;
-// tma: rows are 16-byte aligned and V * element size is a multiple of 16, so
-// tiles move with bulk copies (otherwise with plain loads).
-cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool tma, int grid, size_t smem, cudaStream_t s);
+// aligned: every row starts on a 16-byte boundary, so rows are read with
+// 16-byte vector loads (a row's ragged end element-wise); otherwise element-wise.
+// whole: every CTA's tiles lie in one row (the two halves are streamed side by side)
+cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, bool whole, int grid, size_t smem,
+                          cudaStream_t s);
 cudaError_t launch_prune(const PruneArgs& a, int batch, size_t smem, cudaStream_t s);
-cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool tma, int grid, size_t smem, cudaStream_t s);
+cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid, cudaStream_t s);
 size_t expand_keys_bytes(int max_segments, int support);
 size_t expand_smem_bytes(int max_segments, int support);
 int expand_tile_elems(int dtype);
-size_t verify_stream_smem_bytes();
 int verify_table_width(int K);
-int verify_tile_elems(int dtype);
+int verify_chunks_per_row(int dtype, int V);
+int verify_stream_grid(int sms, int64_t chunks);
+int verify_stream_units(int grid, int64_t chunks);
 
 }  // namespace rheo

@@ -1,20 +1,26 @@
 // verify.cu -- RheoVerification (Algorithm 1) applied layer by layer (Theorem 1).
 //
-// verify_stream_kernel: persistent CTAs stream the B*(N+1) target rows tile by
-// tile (stream.cuh), keeping a running (max, sum exp((l - max) / T)) per
-// thread over each row segment.  The CTA that ends the last segment of a row
-// (arrival counter, never a wait) turns the row into its decision table:
-// lse_T, p at the surviving children, and -- when the row's sampled child
-// survived -- r^ = max(0, p - q~) over the tail that child was drawn from, the
-// residual mass M = 1 - sum_tail min(p, q~), r^ at the children, plus the
-// Philox coins of the node.  Every row is independent, so all tables are built
-// in parallel while the stream is still running.
+// Three launches on the caller's stream:
 //
-// residual_kernel, grid (chunks, B): each CTA stages its request's tables,
-// replays the walk of Algorithm 1 from the root (a few comparisons per level),
-// and takes part in the final draw u* ~ r over V minus the candidate set
-// (Gumbel-max over the stopping row; chunk maxima meet through 64-bit
-// atomicMax, the last CTA of the request writes the bonus token).
+// verify_stream_kernel: every warp streams its own contiguous run of 2 KB
+// chunks of the B*(N+1) target rows (16-byte loads straight into registers,
+// the next chunk in flight while the current one is summed), keeping a running
+// (max, sum exp((l - max) / T)) per lane.  Where a row segment of its run ends
+// the warp reduces that state and writes the segment's partial.  The warps
+// never wait for one another.
+//
+// verify_rows_kernel: one warp per pruned row builds the row's decision table:
+// lse_T from the partials, p at the surviving children and -- when the row's
+// sampled child survived -- r^ = max(0, p - q~) over the tail that child was
+// drawn from, the residual mass M = 1 - sum_tail min(p, q~), r^ at the
+// children, the Philox coins of the node, and the verdict of Algorithm 1 at
+// the node.  A row's verdict depends on nothing but the row itself.
+//
+// residual_kernel, grid (chunks, B): each CTA stages its request's verdicts,
+// replays the walk from the root (a few comparisons per level), and takes part
+// in the final draw u* ~ r over V minus the candidate set (Gumbel-max over the
+// stopping row; chunk maxima meet through 64-bit atomicMax, the last CTA of the
+// request writes the bonus token).
 #include "rheo_device.cuh"
 #include "rheo_kernels.h"
 #include "stream.cuh"
@@ -30,25 +36,21 @@ namespace {
 //   7 .. 7+K+1        p at the children (slot order of the pruned row)
 //   7+K+1 .. 7+2K+2   r^ at the children (p when the sampled child did not survive)
 //   7+2K+2 .. +K+2    coins: draw 0 (sampled child), draw 1+slot (others)
-// A row's verdict depends on nothing but the row itself (Algorithm 1 at one
-// node), so every row gets it in parallel; the walk only follows verdicts.
 constexpr int kTabP = 7;
 __host__ __device__ __forceinline__ int table_width(int K) { return kTabP + 2 * (K + 1) + (K + 2); }
 
-struct RowSmem {
-    int32_t tok[kMaxSupport];    // children tokens
-    int32_t cgen[kMaxSupport];   // children gen ids
-    int32_t tids[kMaxSupport];   // tail ids
-    float tq[kMaxSupport];       // tail q~
-    float lval[2 * kMaxSupport]; // gathered logits: children, then tail
-    int32_t cpos[kMaxSupport];   // tail position of each child (-1: off the tail)
-    float pt[kMaxSupport];       // r^ over the tail
-    float pc[kMaxSupport];       // p at the children
-    float rc[kMaxSupport];       // r^ at the children
-    float coin[kMaxSupport + 2]; // Philox coins of the node
-    float qs;                    // q~ of the sampled child
-    int nc, fc, sc, gen;
-    int64_t e;
+constexpr int kCV = 4;                     // 16-byte vectors per lane per chunk
+constexpr int kChunkBytesW = 32 * kCV * 16;  // bytes one warp takes per step
+constexpr int kRowWarps = 4;               // warps (rows) per CTA of the rows kernel
+
+struct WarpRow {
+    int32_t tok[kMaxSupport];   // children tokens
+    int32_t cgen[kMaxSupport];  // children gen ids
+    int32_t tids[kMaxSupport];  // tail ids
+    float pc[kMaxSupport];      // p at the children
+    float rc[kMaxSupport];      // r^ at the children
+    float pt[kMaxSupport];      // r^ over the tail
+    float coin[kMaxSupport + 2];
 };
 
 __device__ __forceinline__ bool pruned_row_ok(int nc, int fc, int sc, int K, int N) {
@@ -80,232 +82,216 @@ __device__ __forceinline__ FF combine_lse(const float* mu, const float* sm, int 
     return ff_add(ff_div(m, T), ff_log(t));  // m / T + log sum
 }
 
+// one warp: (max, float-float sum of 2^((x - max) c)) of the lanes' (m, s)
+__device__ __forceinline__ FF warp_partition(float m, float s, float c, float& M) {
+    FF v{s, 0.0f};
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o);
+        const FF v2 = ff_shfl_xor(v, o);
+        const float mm = fmaxf(m, m2);
+        const FF x = (m == -INFINITY) ? FF{0.0f, 0.0f} : ff_mul(fast_exp2((m - mm) * c), v);
+        const FF y = (m2 == -INFINITY) ? FF{0.0f, 0.0f} : ff_mul(fast_exp2((m2 - mm) * c), v2);
+        v = ff_add(x, y);
+        m = mm;
+    }
+    M = m;
+    return v;
+}
+
+template <int DT, bool ALIGNED>
+__device__ __forceinline__ void load_chunk(uint4 (&v)[kCV], const char* row, int e0, int V) {
+    using E = Elem<DT>;
+    constexpr int CE = 32 * kCV * E::VEC;
+    const int lane = threadIdx.x & 31;
+    if (ALIGNED && e0 + CE <= V) {
+#pragma unroll
+        for (int j = 0; j < kCV; ++j) v[j] = ld_stream(row + ((int64_t)e0 + (j * 32 + lane) * E::VEC) * E::SIZE);
+        return;
+    }
+#pragma unroll
+    for (int j = 0; j < kCV; ++j) v[j] = load_vec<DT, ALIGNED>(row, (int64_t)e0 + (j * 32 + lane) * E::VEC, V);
+}
+
 }  // namespace
 
-template <int DT, bool TMA>
+template <int DT, bool ALIGNED>
 __global__ void __launch_bounds__(kThreads, 2) verify_stream_kernel(const VerifyArgs a) {
     using E = Elem<DT>;
     using W = Vec<DT>;
     constexpr int VEC = E::VEC;
-    constexpr int TE = kTileBytes / E::SIZE;
-    constexpr int VPT = TE / VEC / kThreads;
+    constexpr int CE = 32 * kCV * VEC;  // elements per chunk
     constexpr float kLog2e = 1.4426950408889634f;
-    extern __shared__ __align__(128) unsigned char dsm[];
-    unsigned char* ring = dsm;
-    __shared__ __align__(8) uint64_t full[kStages];
-    __shared__ BlockScratch bs;
-    __shared__ RowSmem rs;
-
     const Dims& n = a.n;
-    const int tid = threadIdx.x;
-    const int V = n.V, K = n.K, TL = n.TL, NP = n.N + 1;
-    const int tpr = (V + TE - 1) / TE;
-    const TileSplit sp{(int64_t)n.B * NP * tpr, (int)gridDim.x};
-    const int64_t t0 = sp.begin(blockIdx.x), t1 = sp.begin(blockIdx.x + 1);
-    const int TW = table_width(K);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int V = n.V, NP = n.N + 1;
+    const int cpr = n.chunks;
+    const TileSplit sp{(int64_t)n.B * NP * cpr, a.units};
+    const int u = blockIdx.x * kWarps + warp;
+    if (u >= a.units) return;  // units <= chunks: every unit has at least one chunk
+    const int64_t c0 = sp.begin(u), c1 = sp.begin(u + 1);
 
-    if (TMA && tid == 0) {
-        for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
-        mbar_fence_init();
-    }
-    __syncthreads();
-    auto issue = [&](int64_t t) {
-        const int64_t r = t / tpr;
-        const int64_t e0 = (t % tpr) * (int64_t)TE;
-        const unsigned bytes = (unsigned)(min((int64_t)TE, (int64_t)V - e0) * E::SIZE);
-        const int s = (int)((t - t0) % kStages);
-        mbar_arrive_expect_tx(&full[s], bytes);
-        bulk_load(ring + s * kTileBytes, a.logits + r * a.row_stride_bytes + e0 * E::SIZE, bytes, &full[s]);
-    };
-    int64_t issued = t0;
-    if (TMA && tid == 0)
-        for (; issued < min(t1, t0 + kStages); ++issued) issue(issued);
-
+    int64_t r = c0 / cpr;
+    int cc = (int)(c0 % cpr);
+    float c = kLog2e / a.T[r / NP];
     float mu = -INFINITY, sum = 0.0f;
-    bool timed_out = false;
-    int64_t t = t0;
-    for (; t < t1; ++t) {
-        const int64_t r = t / tpr;
-        const int b = (int)(r / NP);
-        const int tt = (int)(t % tpr);
-        const bool seg_first = (t == t0) || (tt == 0);
-        const bool seg_last = (t == t1 - 1) || (tt == tpr - 1);
-        const int s = (int)((t - t0) % kStages);
-        const int64_t e0 = (int64_t)tt * TE;
-        const int ne = (int)min((int64_t)TE, (int64_t)V - e0);
-        unsigned char* tile = ring + s * kTileBytes;
-        const char* row = a.logits + r * a.row_stride_bytes;
-        const float T = a.T[b];
-        bool ok = true;
-        if (TMA) {
-            ok = mbar_wait(&full[s], (unsigned)(((t - t0) / kStages) & 1));
-        } else {
-            for (int e = tid; e < ne; e += kThreads) {
-                const uint32_t w = E::load_scalar(row, e0 + e);
-                if (DT == 0) reinterpret_cast<uint32_t*>(tile)[e] = w;
-                else reinterpret_cast<uint16_t*>(tile)[e] = (uint16_t)w;
-            }
-            __syncthreads();
+    uint4 nxt[kCV];
+    load_chunk<DT, ALIGNED>(nxt, a.logits + r * a.row_stride_bytes, cc * CE, V);
+    for (int64_t t = c0; t < c1; ++t, ++cc) {
+        if (cc == cpr) {
+            cc = 0;
+            ++r;
+            c = kLog2e / a.T[r / NP];
         }
-        if (seg_first) {
-            mu = -INFINITY;
-            sum = 0.0f;
-        }
-        const bool fullt = (ne == TE);
-        uint4 v[VPT];
+        const bool seg_last = (t == c1 - 1) || (cc == cpr - 1);
+        uint4 v[kCV];
 #pragma unroll
-        for (int j = 0; j < VPT; ++j) {
-            v[j] = *reinterpret_cast<const uint4*>(tile + (size_t)(j * kThreads + tid) * 16);
-            if (!fullt) v[j] = W::mask(v[j], ne - (j * kThreads + tid) * VEC);
+        for (int j = 0; j < kCV; ++j) v[j] = nxt[j];
+        if (t + 1 < c1) {
+            const bool wrap = (cc + 1 == cpr);
+            load_chunk<DT, ALIGNED>(nxt, a.logits + (r + (wrap ? 1 : 0)) * a.row_stride_bytes, wrap ? 0 : (cc + 1) * CE, V);
         }
-        // every thread has its values in registers: the stage can be refilled
-        if (!__syncthreads_and(ok)) {
-            timed_out = true;
-            break;
-        }
-        if (TMA && tid == 0 && issued < t1) issue(issued++);
-        const float tmax = fmaxf(fmaxf(W::vmax(v[0]), W::vmax(v[1])), fmaxf(W::vmax(v[2]), W::vmax(v[3])));
-        const float c = kLog2e / T;
+        float tmax = W::vmax(v[0]);
+#pragma unroll
+        for (int j = 1; j < kCV; ++j) tmax = fmaxf(tmax, W::vmax(v[j]));
         if (tmax > mu) {
             if (mu != -INFINITY) sum *= fast_exp2((mu - tmax) * c);
             mu = tmax;
         }
         if (mu != -INFINITY) {
             const float mc = mu * c;
-            sum += (W::vexp(v[0], c, mc) + W::vexp(v[1], c, mc)) + (W::vexp(v[2], c, mc) + W::vexp(v[3], c, mc));
+            float s = 0.0f;
+#pragma unroll
+            for (int j = 0; j < kCV; ++j) s += W::vexp(v[j], c, mc);
+            sum += s;
         }
         if (!seg_last) continue;
+        // ---- end of this warp's segment of row r: its partial ------------------
+        float M;
+        const FF Sw = warp_partition(mu, sum, c, M);
+        if (lane == 0) {
+            const int seg = u - sp.owner(r * cpr);
+            a.seg_mu[r * cpr + seg] = M;
+            a.seg_sum[2 * (r * cpr + seg)] = Sw.hi;
+            a.seg_sum[2 * (r * cpr + seg) + 1] = Sw.lo;
+            if (isnan(Sw.hi) || M == INFINITY) atomicOr(a.status, kStBadLogit);
+        }
+        mu = -INFINITY;
+        sum = 0.0f;
+    }
+}
 
-        // ---- end of segment: partial sums to the workspace ----------------------
-        const int first_owner = sp.owner(r * tpr);
-        const int seg = (int)blockIdx.x - first_owner;
-        const int nseg = sp.owner(r * tpr + tpr - 1) - first_owner + 1;
-        const float Ms = block_max_f32(mu, bs);
-        const FF Ss = block_sum_ff((mu != -INFINITY) ? sum * fast_exp2((mu - Ms) * c) : sum, bs);
-        if (tid == 0) {
-            a.seg_mu[r * tpr + seg] = Ms;
-            a.seg_sum[2 * (r * tpr + seg)] = Ss.hi;
-            a.seg_sum[2 * (r * tpr + seg) + 1] = Ss.lo;
-            if (isnan(Ss.hi) || Ms == INFINITY) atomicOr(a.status, kStBadLogit);
-            if (seg == 0 && (r % NP) == 0 && (!(T > 0.0f) || isinf(T))) atomicOr(a.status, kStBadTemperature);
-        }
-        if (!arrive_last(a.row_ticket + r, (unsigned)nseg, bs)) continue;
+// One warp per pruned row: the row's decision table (Algorithm 1 at the node).
+template <int DT>
+__global__ void __launch_bounds__(32 * kRowWarps) verify_rows_kernel(const VerifyArgs a) {
+    using E = Elem<DT>;
+    __shared__ WarpRow wrs[kRowWarps];
+    const Dims& n = a.n;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int V = n.V, K = n.K, TL = n.TL, NP = n.N + 1;
+    const int64_t r = (int64_t)blockIdx.x * kRowWarps + warp;
+    if (r >= (int64_t)n.B * NP) return;
+    WarpRow& w = wrs[warp];
+    const int b = (int)(r / NP);
+    const int cpr = n.chunks;
+    const int TW = table_width(K);
+    const TileSplit sp{(int64_t)n.B * NP * cpr, a.units};
+    const int nseg = sp.owner(r * cpr + cpr - 1) - sp.owner(r * cpr) + 1;
+    const float T = a.T[b];
+    const FF lse = combine_lse(a.seg_mu + r * cpr, a.seg_sum + 2 * r * cpr, nseg, T);
+    float* tab = a.table + r * TW;
 
-        // ---- last segment of row r: its decision table ----------------------------
-        float* tab = a.table + r * TW;
-        if (tid < 32) {
-            const FF l2 = combine_lse(a.seg_mu + r * tpr, a.seg_sum + 2 * r * tpr, nseg, T);
-            if (tid == 0) {
-                tab[3] = l2.hi;
-                tab[4] = l2.lo;
-                if (a.row_lse) a.row_lse[r] = __fadd_rn(l2.hi, l2.lo);
-                if (!(l2.hi > -INFINITY)) atomicOr(a.status, kStEmptyRow);
-                int nc = a.pr.n_child[r], fc = a.pr.first_child[r], sc = a.pr.sampled_child[r];
-                if (!pruned_row_ok(nc, fc, sc, K, n.N)) {
-                    atomicOr(a.status, kStInternal);
-                    nc = 0, sc = -1;
-                }
-                rs.nc = nc;
-                rs.fc = fc;
-                rs.sc = sc;
-                rs.gen = a.pr.gen_id[r];
-                rs.e = (sc >= 0) ? expansion_of_child(K, a.pr.gen_id[(int64_t)b * NP + sc], n.G1, n.E) : 0;
-            }
-        }
-        __syncthreads();
-        const int nc = rs.nc, fc = rs.fc, sc = rs.sc;
-        const FF lse{tab[3], tab[4]};
-        const int64_t q0 = ((int64_t)b * n.E + rs.e) * TL;
-        // gather: children tokens, then (sampled child alive) the tail of its draw
-        if (tid < nc) {
-            rs.tok[tid] = a.pr.token[(int64_t)b * NP + fc + tid];
-            rs.cgen[tid] = a.pr.gen_id[(int64_t)b * NP + fc + tid];
-        }
-        if (sc >= 0 && tid < TL) {
-            rs.tids[tid] = a.tree.tail_ids[q0 + tid];
-            rs.tq[tid] = a.tree.tail_q[q0 + tid];
-        }
-        __syncthreads();
-        for (int i = tid; i < nc + (sc >= 0 ? TL : 0); i += kThreads) {
-            const int tok = (i < nc) ? rs.tok[i] : rs.tids[i - nc];
-            rs.lval[i] = (tok >= 0 && tok < V) ? E::value(E::load_scalar(row, tok)) : -INFINITY;
-        }
-        __syncthreads();
-        const uint64_t seed = a.seed[b], off = a.offset[b];
-        float ov = 0.0f;
-        if (sc >= 0 && tid < TL) {
-            const float pt = exp_scaled_minus(rs.lval[nc + tid], T, lse);
-            const float qi = rs.tq[tid];
+    int nc = a.pr.n_child[r], fc = a.pr.first_child[r], sc = a.pr.sampled_child[r];
+    if (!pruned_row_ok(nc, fc, sc, K, n.N)) {
+        if (lane == 0) atomicOr(a.status, kStInternal);
+        nc = 0;
+        sc = -1;
+    }
+    if (lane == 0) {
+        tab[3] = lse.hi;
+        tab[4] = lse.lo;
+        if (a.row_lse) a.row_lse[r] = __fadd_rn(lse.hi, lse.lo);
+        if (!(lse.hi > -INFINITY)) atomicOr(a.status, kStEmptyRow);
+        if ((r % NP) == 0 && (!(T > 0.0f) || isinf(T))) atomicOr(a.status, kStBadTemperature);
+    }
+    const int gen = a.pr.gen_id[r];
+    const int64_t pb = (int64_t)b * NP;
+    const int64_t e = (sc >= 0) ? expansion_of_child(K, a.pr.gen_id[pb + sc], n.G1, n.E) : 0;
+    const int64_t q0 = ((int64_t)b * n.E + e) * TL;
+    const char* row = a.logits + r * a.row_stride_bytes;
+    auto logit = [&](int tok) -> float { return (tok >= 0 && tok < V) ? E::value(E::load_scalar(row, tok)) : -INFINITY; };
+
+    for (int i = lane; i < nc; i += 32) {
+        const int tok = a.pr.token[pb + fc + i];
+        w.tok[i] = tok;
+        w.cgen[i] = a.pr.gen_id[pb + fc + i];
+        w.pc[i] = exp_scaled_minus(logit(tok), T, lse);
+    }
+    // the tail of the sampled child's draw, when that child survived
+    FF ov{0.0f, 0.0f};
+    if (sc >= 0)
+        for (int i = lane; i < TL; i += 32) {
+            const int tok = a.tree.tail_ids[q0 + i];
+            const float qi = a.tree.tail_q[q0 + i];
+            const float pt = exp_scaled_minus(logit(tok), T, lse);
             const float d = __fsub_rn(pt, qi);
             const float rh = d > 0.0f ? d : 0.0f;
-            rs.pt[tid] = rh;
-            a.rhat_tail[r * TL + tid] = rh;
-            ov = fminf(pt, qi);
+            w.tids[i] = tok;
+            w.pt[i] = rh;
+            a.rhat_tail[r * TL + i] = rh;
+            ov = ff_add(ov, fminf(pt, qi));
         }
-        if (tid < nc) {
-            int pos = -1;
-            if (sc >= 0)
-                for (int i = 0; i < TL; ++i)
-                    if (rs.tids[i] == rs.tok[tid]) pos = i;
-            rs.cpos[tid] = pos;
-        }
-        const FF overlap = block_sum_ff(ov, bs);  // also orders the rs writes above
-        if (tid < nc) {
-            const float p = exp_scaled_minus(rs.lval[tid], T, lse);
-            const float rh = (rs.cpos[tid] >= 0) ? rs.pt[rs.cpos[tid]] : p;
-            rs.pc[tid] = p;
-            rs.rc[tid] = rh;
-            tab[kTabP + tid] = p;
-            tab[kTabP + (K + 1) + tid] = rh;
-        }
-        if (tid < K + 2) {
-            const float u = uniform(seed, off, kTagVerify, rs.gen, (uint64_t)tid);
-            rs.coin[tid] = u;
-            tab[kTabP + 2 * (K + 1) + tid] = u;
-        }
-        if (tid == kThreads - 1) rs.qs = (sc >= 0) ? a.tree.qtilde[(int64_t)b * n.G1 + rs.cgen[sc - fc]] : 0.0f;
-        __syncthreads();
-        if (tid == 0) {
-            // Algorithm 1 at this node: stochastic first, then recursive rejection in slot order
-            const float qs = rs.qs;
-            FF M{1.0f, 0.0f};
-            int acc = -1, use_tail = 0;
-            if (sc >= 0) {
-                if (__fmul_rn(rs.coin[0], qs) <= rs.pc[sc - fc]) {
-                    acc = sc;
-                } else {
-                    M = ff_add(FF{1.0f, 0.0f}, ff_neg(overlap));
-                    use_tail = 1;
-                }
-            }
-            const FF M0 = M;
-            if (acc < 0)
-                for (int c2 = 0; c2 < nc; ++c2) {
-                    if (fc + c2 == sc) continue;
-                    const float eta = rs.coin[1 + slot_of(K, rs.cgen[c2])];
-                    const float rv = use_tail ? rs.rc[c2] : rs.pc[c2];
-                    if (ff_le(ff_mul(eta, M), rv)) {  // eta * M <= r^(u_i)
-                        acc = fc + c2;
-                        break;
-                    }
-                    M = ff_add(M, -rv);
-                }
-            tab[0] = M0.hi;
-            tab[1] = M0.lo;
-            tab[2] = qs;
-            tab[5] = (float)use_tail;
-            tab[6] = (float)acc;
-        }
-        __syncthreads();
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) ov = ff_add(ov, ff_shfl_xor(ov, o));
+    const uint64_t seed = a.seed[b], off = a.offset[b];
+    for (int i = lane; i < K + 2; i += 32) {
+        const float u = uniform(seed, off, kTagVerify, gen, (uint64_t)i);
+        w.coin[i] = u;
+        tab[kTabP + 2 * (K + 1) + i] = u;
     }
-
-    if (timed_out) {
-        if (tid == 0) {
-            atomicOr(a.status, kStTimeout);
-            for (int64_t u = t; u < issued; ++u)
-                mbar_wait(&full[(int)((u - t0) % kStages)], (unsigned)(((u - t0) / kStages) & 1));
+    __syncwarp();
+    for (int i = lane; i < nc; i += 32) {
+        int pos = -1;
+        if (sc >= 0)
+            for (int j = 0; j < TL; ++j)
+                if (w.tids[j] == w.tok[i]) pos = j;
+        const float p = w.pc[i];
+        const float rh = (pos >= 0) ? w.pt[pos] : p;
+        w.rc[i] = rh;
+        tab[kTabP + i] = p;
+        tab[kTabP + (K + 1) + i] = rh;
+    }
+    __syncwarp();
+    if (lane == 0) {
+        // Algorithm 1 at this node: stochastic first, then recursive rejection in slot order
+        const float qs = (sc >= 0) ? a.tree.qtilde[(int64_t)b * n.G1 + w.cgen[sc - fc]] : 0.0f;
+        FF M{1.0f, 0.0f};
+        int acc = -1, use_tail = 0;
+        if (sc >= 0) {
+            if (__fmul_rn(w.coin[0], qs) <= w.pc[sc - fc]) {
+                acc = sc;
+            } else {
+                M = ff_add(FF{1.0f, 0.0f}, ff_neg(ov));
+                use_tail = 1;
+            }
         }
-        __syncthreads();
+        const FF M0 = M;
+        if (acc < 0)
+            for (int c2 = 0; c2 < nc; ++c2) {
+                if (fc + c2 == sc) continue;
+                const float eta = w.coin[1 + slot_of(K, w.cgen[c2])];
+                const float rv = use_tail ? w.rc[c2] : w.pc[c2];
+                if (ff_le(ff_mul(eta, M), rv)) {  // eta * M <= r^(u_i)
+                    acc = fc + c2;
+                    break;
+                }
+                M = ff_add(M, -rv);
+            }
+        tab[0] = M0.hi;
+        tab[1] = M0.lo;
+        tab[2] = qs;
+        tab[5] = (float)use_tail;
+        tab[6] = (float)acc;
     }
 }
 
@@ -453,27 +439,41 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     }
 }
 
-cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool tma, int grid, size_t smem, cudaStream_t s) {
+cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid, cudaStream_t s) {
     auto go_stream = [&](auto kern) {
-        cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (err != cudaSuccess) return err;
-        kern<<<grid, kThreads, smem, s>>>(a);
+        kern<<<grid, kThreads, 0, s>>>(a);
         return cudaGetLastError();
     };
     cudaError_t err;
-    if (dtype == 1) err = tma ? go_stream(verify_stream_kernel<1, true>) : go_stream(verify_stream_kernel<1, false>);
-    else err = tma ? go_stream(verify_stream_kernel<0, true>) : go_stream(verify_stream_kernel<0, false>);
+    if (dtype == 1) err = aligned ? go_stream(verify_stream_kernel<1, true>) : go_stream(verify_stream_kernel<1, false>);
+    else err = aligned ? go_stream(verify_stream_kernel<0, true>) : go_stream(verify_stream_kernel<0, false>);
     if (err != cudaSuccess) return err;
+    const int64_t rows = (int64_t)a.n.B * (a.n.N + 1);
+    const int g1 = (int)((rows + kRowWarps - 1) / kRowWarps);
+    if (dtype == 1) verify_rows_kernel<1><<<g1, 32 * kRowWarps, 0, s>>>(a);
+    else verify_rows_kernel<0><<<g1, 32 * kRowWarps, 0, s>>>(a);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
     const dim3 g2((a.n.V + kResChunk - 1) / kResChunk, a.n.B);
-    auto go_res = [&](auto kern) {
-        kern<<<g2, kThreads, 0, s>>>(a);
-        return cudaGetLastError();
-    };
-    return dtype == 1 ? go_res(residual_kernel<1>) : go_res(residual_kernel<0>);
+    if (dtype == 1) residual_kernel<1><<<g2, kThreads, 0, s>>>(a);
+    else residual_kernel<0><<<g2, kThreads, 0, s>>>(a);
+    return cudaGetLastError();
 }
 
-size_t verify_stream_smem_bytes() { return (size_t)kStages * kTileBytes; }
 int verify_table_width(int K) { return table_width(K); }
-int verify_tile_elems(int dtype) { return kTileBytes / (dtype == 1 ? 2 : 4); }
+int verify_chunks_per_row(int dtype, int V) {
+    const int ce = kChunkBytesW / (dtype == 1 ? 2 : 4);
+    return (V + ce - 1) / ce;
+}
+// stream grid: two CTAs per SM, no more CTAs than needed for one chunk per warp
+int verify_stream_grid(int sms, int64_t chunks) {
+    const int64_t g = 2 * (int64_t)sms;
+    const int64_t need = (chunks + kWarps - 1) / kWarps;
+    return (int)(g < need ? g : need);
+}
+// stream units (warps with work): never more than chunks, so none is empty
+int verify_stream_units(int grid, int64_t chunks) {
+    const int64_t u = (int64_t)grid * kWarps;
+    return (int)(u < chunks ? u : chunks);
+}
 
 }  // namespace rheo

@@ -320,6 +320,7 @@ __device__ __noinline__ void insert_rounds(unsigned long long* region, int& cnt,
 
 template <int DT, bool ALIGNED, int NS>
 __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const ExpandArgs a) {
+    grid_dependency_begin();
     using E = Elem<DT>;
     using W = Vec<DT>;
     constexpr int VEC = E::VEC;
@@ -793,8 +794,7 @@ cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, bool who
     auto go = [&](auto kern) {
         cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (err != cudaSuccess) return err;
-        kern<<<grid, kThreads, smem, s>>>(a);
-        return cudaGetLastError();
+        return launch_dependent(kern, dim3(grid), dim3(kThreads), smem, s, a);
     };
     if (whole) {
         if (dtype == 1) return aligned ? go(expand_kernel<1, true, 2>) : go(expand_kernel<1, false, 2>);

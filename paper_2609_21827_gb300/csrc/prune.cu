@@ -12,6 +12,7 @@
 namespace rheo {
 
 __global__ void __launch_bounds__(kThreads) prune_kernel(const PruneArgs a) {
+    grid_dependency_begin();
     extern __shared__ __align__(16) unsigned char psm[];
     __shared__ BlockScratch bs;
     __shared__ unsigned hist[kRadixBins];
@@ -98,7 +99,8 @@ cudaError_t launch_prune(const PruneArgs& a, int batch, size_t smem, cudaStream_
         const cudaError_t err = cudaFuncSetAttribute(prune_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (err != cudaSuccess) return err;
     }
-    prune_kernel<<<batch, kThreads, smem, s>>>(a);
+    const cudaError_t err = launch_dependent(prune_kernel, dim3(batch), dim3(kThreads), smem, s, a);
+    if (err != cudaSuccess) return err;
     return cudaGetLastError();
 }
 

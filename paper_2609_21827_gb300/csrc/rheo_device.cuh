@@ -20,6 +20,15 @@ constexpr int kCandCap = 2048;                         // per-chunk candidate bu
 constexpr int kMaxVocab = 262144;
 constexpr int kMaxNodes = 16384;
 
+// Programmatic dependent launch: every kernel of the path first waits until
+// the grid before it on the stream has completed and its writes are visible
+// (a no-op when launched without the programmatic attribute), then lets the
+// next grid start launching, so launch latency overlaps the end of this one.
+__device__ __forceinline__ void grid_dependency_begin() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 enum : uint32_t {
     kStBadLogit = 1u,
     kStEmptyRow = 2u,

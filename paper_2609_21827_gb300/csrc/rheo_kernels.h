@@ -87,6 +87,24 @@ struct VerifyArgs {
     unsigned* res_ticket;           // [B]
 };
 
+// Launch with the programmatic stream serialization attribute: the kernel may
+// start launching while the previous kernel on the stream finishes; kernels
+// call grid_dependency_begin() before touching global memory.
+template <class... P, class... A>
+cudaError_t launch_dependent(void (*kern)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, A&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<A&&>(args)...);
+}
+
 // Host launchers, defined next to their kernels.  dtype: 0 fp32, 1 bf16;
 // aligned: every row starts on a 16-byte boundary, so rows are read with
 // 16-byte vector loads (a row's ragged end element-wise); otherwise element-wise.

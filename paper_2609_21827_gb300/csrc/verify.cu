@@ -117,6 +117,7 @@ __device__ __forceinline__ void load_chunk(uint4 (&v)[kCV], const char* row, int
 
 template <int DT, bool ALIGNED>
 __global__ void __launch_bounds__(kThreads, 2) verify_stream_kernel(const VerifyArgs a) {
+    grid_dependency_begin();
     using E = Elem<DT>;
     using W = Vec<DT>;
     constexpr int VEC = E::VEC;
@@ -184,6 +185,7 @@ __global__ void __launch_bounds__(kThreads, 2) verify_stream_kernel(const Verify
 // One warp per pruned row: the row's decision table (Algorithm 1 at the node).
 template <int DT>
 __global__ void __launch_bounds__(32 * kRowWarps) verify_rows_kernel(const VerifyArgs a) {
+    grid_dependency_begin();
     using E = Elem<DT>;
     __shared__ WarpRow wrs[kRowWarps];
     const Dims& n = a.n;
@@ -198,10 +200,11 @@ __global__ void __launch_bounds__(32 * kRowWarps) verify_rows_kernel(const Verif
     const TileSplit sp{(int64_t)n.B * NP * cpr, a.units};
     const int nseg = sp.owner(r * cpr + cpr - 1) - sp.owner(r * cpr) + 1;
     const float T = a.T[b];
+    int nc = a.pr.n_child[r], fc = a.pr.first_child[r], sc = a.pr.sampled_child[r];
+    const int gen = a.pr.gen_id[r];
     const FF lse = combine_lse(a.seg_mu + r * cpr, a.seg_sum + 2 * r * cpr, nseg, T);
     float* tab = a.table + r * TW;
 
-    int nc = a.pr.n_child[r], fc = a.pr.first_child[r], sc = a.pr.sampled_child[r];
     if (!pruned_row_ok(nc, fc, sc, K, n.N)) {
         if (lane == 0) atomicOr(a.status, kStInternal);
         nc = 0;
@@ -214,7 +217,6 @@ __global__ void __launch_bounds__(32 * kRowWarps) verify_rows_kernel(const Verif
         if (!(lse.hi > -INFINITY)) atomicOr(a.status, kStEmptyRow);
         if ((r % NP) == 0 && (!(T > 0.0f) || isinf(T))) atomicOr(a.status, kStBadTemperature);
     }
-    const int gen = a.pr.gen_id[r];
     const int64_t pb = (int64_t)b * NP;
     const int64_t e = (sc >= 0) ? expansion_of_child(K, a.pr.gen_id[pb + sc], n.G1, n.E) : 0;
     const int64_t q0 = ((int64_t)b * n.E + e) * TL;
@@ -250,11 +252,27 @@ __global__ void __launch_bounds__(32 * kRowWarps) verify_rows_kernel(const Verif
         tab[kTabP + 2 * (K + 1) + i] = u;
     }
     __syncwarp();
+    // tail position of the sampled child: fills sit at the next ranks, Y skipped
+    int ypos = -1;
+    if (sc >= 0) {
+        const int ytok = w.tok[sc - fc];
+        for (int i0 = 0; i0 < TL && ypos < 0; i0 += 32) {
+            const unsigned hit = __ballot_sync(0xFFFFFFFFu, i0 + lane < TL && w.tids[i0 + lane] == ytok);
+            if (hit) ypos = i0 + __ffs(hit) - 1;
+        }
+    }
     for (int i = lane; i < nc; i += 32) {
         int pos = -1;
-        if (sc >= 0)
-            for (int j = 0; j < TL; ++j)
-                if (w.tids[j] == w.tok[i]) pos = j;
+        if (sc >= 0) {
+            const int j = slot_of(K, w.cgen[i]);
+            const int qf = j - n.m - 1;
+            pos = (j < n.m) ? -1 : (j == n.m) ? ypos : qf + (qf >= ypos ? 1 : 0);
+            if (pos >= TL || (pos >= 0 && w.tids[pos] != w.tok[i]) || (pos < 0 && j >= n.m)) {
+                pos = -1;  // not the layout of the expansion: search the tail
+                for (int q = 0; q < TL; ++q)
+                    if (w.tids[q] == w.tok[i]) pos = q;
+            }
+        }
         const float p = w.pc[i];
         const float rh = (pos >= 0) ? w.pt[pos] : p;
         w.rc[i] = rh;
@@ -298,13 +316,21 @@ __global__ void __launch_bounds__(32 * kRowWarps) verify_rows_kernel(const Verif
 // ---------------------------------------------------------------------------
 // walk + final draw
 // ---------------------------------------------------------------------------
-constexpr int kResChunk = 2048;  // elements of the stopping row per residual CTA
+constexpr int kResChunk = 4096;  // elements of the stopping row per residual CTA
+constexpr int kResPer = kResChunk / kThreads;  // consecutive elements per thread
 constexpr int kStageRows = 1024; // pruned rows whose verdicts the walk stages in shared memory
+
+__device__ __forceinline__ unsigned long long pack_key(float key, int64_t id) {
+    return ((unsigned long long)ord_f32(key) << 32) | (0xFFFFFFFFu - (uint32_t)id);
+}
 
 template <int DT>
 __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) {
+    grid_dependency_begin();
     using E = Elem<DT>;
+    static_assert(kResPer % 4 == 0, "whole Philox blocks per thread");
     __shared__ BlockScratch bs;
+    __shared__ Red red;
     __shared__ uint32_t excl_bits[kResChunk / 32];
     __shared__ uint32_t tail_bits[kResChunk / 32];
     __shared__ int s_stop, s_len;
@@ -318,10 +344,15 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     const int V = n.V, K = n.K, TL = n.TL, NP = n.N + 1, D = n.D;
     const int TW = table_width(K);
     const int64_t pb = (int64_t)b * NP;
+    int par = 0;
     // the walk follows the per-row verdicts from the root (staged when they fit)
     const bool staged = NP <= kStageRows;
     if (staged)
         for (int i = tid; i < NP; i += kThreads) s_verdict[i] = (int)__ldcg(a.table + (pb + i) * TW + 6);
+    for (int i = tid; i < kResChunk / 32; i += kThreads) {
+        excl_bits[i] = 0u;
+        tail_bits[i] = 0u;
+    }
     __syncthreads();
     if (tid == 0) {
         int u = 0, len = 0;
@@ -365,8 +396,6 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     const char* row = a.logits + rowg * a.row_stride_bytes;
     const int64_t e_lo = (int64_t)k * kResChunk;
 
-    for (int i = tid; i < kResChunk / 32; i += kThreads) { excl_bits[i] = 0u; tail_bits[i] = 0u; }
-    __syncthreads();
     for (int c = tid; c < nc_ok; c += kThreads) {
         const int tok = a.pr.token[pb + fc + c];
         if (tok >= e_lo && tok < e_lo + kResChunk)
@@ -380,35 +409,28 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
         }
     __syncthreads();
 
-    // keys: 0 -> r^ over V minus the candidates; 1 -> p over V minus the
-    // candidates; 2 -> p over V (1 and 2 only matter after rounding dead ends)
-    unsigned long long best[3] = {0ull, 0ull, 0ull};
-    auto offer = [&](int w, float key, int64_t id) {
-        if (key > -INFINITY) {
-            const unsigned long long pk = ((unsigned long long)ord_f32(key) << 32) | (0xFFFFFFFFu - (uint32_t)id);
-            best[w] = pk > best[w] ? pk : best[w];
-        }
-    };
+    // key of the draw from r: log r^ + g on the tail (after a rejection), log p + g
+    // elsewhere, over V minus the candidates
+    unsigned long long best = 0ull;
     {
-        // each thread: 8 consecutive elements, two Philox blocks
-        const int64_t e0 = e_lo + (int64_t)tid * 8;
-        if (e0 < V) {
-            uint4 rnd[2];
-            rnd[0] = philox_block(seed, off, kTagResidual, gen_u, (uint64_t)(e0 >> 2));
-            rnd[1] = philox_block(seed, off, kTagResidual, gen_u, (uint64_t)(e0 >> 2) + 1);
+        const int64_t e0 = e_lo + (int64_t)tid * kResPer;
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const int64_t id = e0 + i;
+        for (int h = 0; h < kResPer / 4; ++h) {
+            if (e0 + 4 * h >= V) break;
+            const uint4 rnd = philox_block(seed, off, kTagResidual, gen_u, (uint64_t)((e0 >> 2) + h));
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int64_t id = e0 + 4 * h + i;
                 if (id >= V) break;
-                const float x = E::value(E::load_scalar(row, id));
-                const float g = gumbel(u01(word_of(rnd[i >> 2], i & 3)));
-                const float tv = __fdiv_rn(x, T);
-                const float fb = __fadd_rn(tv, g);
-                offer(2, fb, id);
                 const int li = (int)(id - e_lo);
-                if ((excl_bits[li >> 5] >> (li & 31)) & 1u) continue;
-                offer(1, fb, id);
-                if (!((tail_bits[li >> 5] >> (li & 31)) & 1u)) offer(0, __fadd_rn(__fsub_rn(tv, lse), g), id);
+                if (((excl_bits[li >> 5] | tail_bits[li >> 5]) >> (li & 31)) & 1u) continue;
+                const float x = E::value(E::load_scalar(row, id));
+                const float g = gumbel(u01(word_of(rnd, i)));
+                const float key = __fadd_rn(__fsub_rn(__fdiv_rn(x, T), lse), g);
+                if (key > -INFINITY) {
+                    const unsigned long long pk = pack_key(key, id);
+                    best = pk > best ? pk : best;
+                }
             }
         }
     }
@@ -422,27 +444,48 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
             const float rv = __ldcg(a.rhat_tail + rowg * TL + i);
             if (!(rv > 0.0f)) continue;
             const float g = gumbel(uniform(seed, off, kTagResidual, gen_u, (uint64_t)tok));
-            offer(0, __fadd_rn(logf(rv), g), tok);
+            const float key = __fadd_rn(logf(rv), g);
+            if (key > -INFINITY) {
+                const unsigned long long pk = pack_key(key, tok);
+                best = pk > best ? pk : best;
+            }
         }
-    for (int w = 0; w < 3; ++w) {
-        const unsigned long long m = block_max_u64(best[w], bs);
-        if (tid == 0 && m) atomicMax(a.res_best + (int64_t)b * 3 + w, m);
+    {
+        const unsigned long long m = red_max_u64(best, red, par);
+        if (tid == 0 && m) atomicMax(a.res_best + (int64_t)b * 3, m);
     }
-    if (!arrive_last(a.res_ticket + b, gridDim.x, bs)) return;
+    if (!arrive_last(a.res_ticket + b, gridDim.x * gridDim.z, bs)) return;
+    unsigned long long m = __ldcg(a.res_best + (int64_t)b * 3);
+    if (!m) {
+        // rounding left no mass in r: draw from p over V minus the candidates, else
+        // over V (one CTA sweeps the whole row; this only follows dead ends)
+        unsigned long long b1 = 0ull, b2 = 0ull;
+        for (int64_t id = tid; id < V; id += kThreads) {
+            bool ex = false;
+            for (int c = 0; c < nc_ok; ++c) ex |= (a.pr.token[pb + fc + c] == id);
+            const float x = E::value(E::load_scalar(row, id));
+            const float g = gumbel(uniform(seed, off, kTagResidual, gen_u, (uint64_t)id));
+            const float key = __fadd_rn(__fdiv_rn(x, T), g);
+            if (key > -INFINITY) {
+                const unsigned long long pk = pack_key(key, id);
+                b2 = pk > b2 ? pk : b2;
+                if (!ex) b1 = pk > b1 ? pk : b1;
+            }
+        }
+        const unsigned long long m1 = red_max_u64(b1, red, par);
+        const unsigned long long m2 = red_max_u64(b2, red, par);
+        m = m1 ? m1 : m2;
+    }
     if (tid == 0) {
-        unsigned long long m = __ldcg(a.res_best + (int64_t)b * 3 + 0);
-        if (!m) m = __ldcg(a.res_best + (int64_t)b * 3 + 1);
-        if (!m) m = __ldcg(a.res_best + (int64_t)b * 3 + 2);
         a.bonus_token[b] = m ? (int32_t)(0xFFFFFFFFu - (uint32_t)m) : -1;
         if (!m) atomicOr(a.status, kStEmptyRow);
-        for (int w = 0; w < 3; ++w) a.res_best[(int64_t)b * 3 + w] = 0ull;  // ready for the next call
+        a.res_best[(int64_t)b * 3] = 0ull;  // ready for the next call
     }
 }
 
 cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid, cudaStream_t s) {
     auto go_stream = [&](auto kern) {
-        kern<<<grid, kThreads, 0, s>>>(a);
-        return cudaGetLastError();
+        return launch_dependent(kern, dim3(grid), dim3(kThreads), 0, s, a);
     };
     cudaError_t err;
     if (dtype == 1) err = aligned ? go_stream(verify_stream_kernel<1, true>) : go_stream(verify_stream_kernel<1, false>);
@@ -450,13 +493,12 @@ cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid
     if (err != cudaSuccess) return err;
     const int64_t rows = (int64_t)a.n.B * (a.n.N + 1);
     const int g1 = (int)((rows + kRowWarps - 1) / kRowWarps);
-    if (dtype == 1) verify_rows_kernel<1><<<g1, 32 * kRowWarps, 0, s>>>(a);
-    else verify_rows_kernel<0><<<g1, 32 * kRowWarps, 0, s>>>(a);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    err = (dtype == 1) ? launch_dependent(verify_rows_kernel<1>, dim3(g1), dim3(32 * kRowWarps), 0, s, a)
+                       : launch_dependent(verify_rows_kernel<0>, dim3(g1), dim3(32 * kRowWarps), 0, s, a);
+    if (err != cudaSuccess) return err;
     const dim3 g2((a.n.V + kResChunk - 1) / kResChunk, a.n.B);
-    if (dtype == 1) residual_kernel<1><<<g2, kThreads, 0, s>>>(a);
-    else residual_kernel<0><<<g2, kThreads, 0, s>>>(a);
-    return cudaGetLastError();
+    return (dtype == 1) ? launch_dependent(residual_kernel<1>, g2, dim3(kThreads), 0, s, a)
+                        : launch_dependent(residual_kernel<0>, g2, dim3(kThreads), 0, s, a);
 }
 
 int verify_table_width(int K) { return table_width(K); }

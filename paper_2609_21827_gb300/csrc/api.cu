@@ -43,7 +43,8 @@ bool valid(const rheo_config* c) {
 
 struct Layout {
     size_t status, ex_row_ticket, ex_req_ticket, ex_mu, ex_sum, ex_keys;
-    size_t v_mu, v_sum, v_table, v_rhat, r_best, r_ticket;
+    size_t v_mu, v_sum, v_row_ticket, v_hdr, v_child, v_tids, v_tq, v_cx, v_tx, v_coin, v_table, v_rhat, r_best,
+        r_ticket;
     size_t total;
 };
 
@@ -64,6 +65,14 @@ Layout layout(const rheo_config& c) {
     L.ex_keys = take(sizeof(unsigned long long) * B * F * P * S);
     L.v_mu = take(sizeof(float) * B * NP * VC);
     L.v_sum = take(2 * sizeof(float) * B * NP * VC);
+    L.v_row_ticket = take(sizeof(unsigned) * B * NP);
+    L.v_hdr = take(sizeof(int) * B * NP * 8);
+    L.v_child = take(sizeof(int) * B * NP * (c.K + 1) * 3);
+    L.v_tids = take(sizeof(int) * B * NP * TL);
+    L.v_tq = take(sizeof(float) * B * NP * TL);
+    L.v_cx = take(2 * sizeof(float) * B * NP * (c.K + 1));
+    L.v_tx = take(2 * sizeof(float) * B * NP * TL);
+    L.v_coin = take(sizeof(float) * B * NP * (c.K + 2));
     L.v_table = take(sizeof(float) * B * NP * verify_table_width(c.K));
     L.v_rhat = take(sizeof(float) * B * NP * TL);
     L.r_best = take(sizeof(unsigned long long) * B * 3);
@@ -233,6 +242,14 @@ extern "C" int rheo_verify(const rheo_config* cfg, const void* logits, int64_t r
     a.status = at<unsigned>(ws, L.status);
     a.seg_mu = at<float>(ws, L.v_mu);
     a.seg_sum = at<float>(ws, L.v_sum);
+    a.row_ticket = at<unsigned>(ws, L.v_row_ticket);
+    a.rec_hdr = at<int>(ws, L.v_hdr);
+    a.rec_child = at<int>(ws, L.v_child);
+    a.rec_tids = at<int>(ws, L.v_tids);
+    a.rec_tq = at<float>(ws, L.v_tq);
+    a.rec_cx = at<float>(ws, L.v_cx);
+    a.rec_tx = at<float>(ws, L.v_tx);
+    a.rec_coin = at<float>(ws, L.v_coin);
     a.table = at<float>(ws, L.v_table);
     a.rhat_tail = at<float>(ws, L.v_rhat);
     a.res_best = at<unsigned long long>(ws, L.r_best);

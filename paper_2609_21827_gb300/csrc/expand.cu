@@ -433,22 +433,17 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
     // own at offsets from a warp scan.
     auto tile_candidates = [&](const uint4 (&v)[kVPT], const float (&vm)[kVPT], int e0, int ne) {
         const float thv = E::threshold_value((uint32_t)(theta >> 32));
+        // the bound in the element's own format (bf16: a pair), compared packed
+        const uint32_t t2 = (DT == 0) ? __float_as_uint(thv)
+                                      : ((__float_as_uint(thv) >> 16) | (__float_as_uint(thv) & 0xFFFF0000u));
         uint32_t pend = 0u;
 #pragma unroll
-        for (int j = 0; j < kVPT; ++j)
-            if (vm[j] >= thv) {
-                if (ne == TE) {
-#pragma unroll
-                    for (int i = 0; i < VEC; ++i)
-                        pend |= (E::value(E::raw(v[j], i)) >= thv) ? (1u << (j * VEC + i)) : 0u;
-                } else {
-#pragma unroll
-                    for (int i = 0; i < VEC; ++i) {
-                        const bool in = (j * kThreads + tid) * VEC + i < ne;
-                        pend |= (in && E::value(E::raw(v[j], i)) >= thv) ? (1u << (j * VEC + i)) : 0u;
-                    }
-                }
-            }
+        for (int j = 0; j < kVPT; ++j) {
+            uint32_t bits = W::ge_bits(v[j], t2);
+            const int left = ne - (j * kThreads + tid) * VEC;  // elements of this vector inside the tile
+            if (left < VEC) bits &= (left > 0) ? ((1u << left) - 1u) : 0u;
+            pend |= bits << (j * VEC);
+        }
         if (!__any_sync(0xFFFFFFFFu, pend != 0u)) return;
 #pragma unroll
         for (int j = 0; j < kVPT; ++j) wspill[j * 32 + lane] = v[j];

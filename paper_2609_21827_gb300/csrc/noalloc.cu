@@ -51,7 +51,8 @@ size_t up256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 // the verification part of the workspace layout, laid out in the static array
 struct StaticLayout {
-    size_t status, mu, sum, table, rhat, best, res_ticket, total, clear_end;
+    size_t status, mu, sum, row_ticket, hdr, child, tids, tq, cx, tx, coin, table, rhat, best, res_ticket, total,
+        clear_end;
 };
 
 StaticLayout static_layout(const rheo_config& c) {
@@ -62,6 +63,7 @@ StaticLayout static_layout(const rheo_config& c) {
     auto take = [&](size_t bytes) { size_t at = o; o = up256(o + bytes); return at; };
     // everything that must start at zero first, so one memset clears it
     L.status = take(sizeof(unsigned));
+    L.row_ticket = take(sizeof(unsigned) * B * NP);
     L.best = take(sizeof(unsigned long long) * B * 3);
     L.res_ticket = take(sizeof(unsigned) * B);
     L.clear_end = o;
@@ -69,6 +71,13 @@ StaticLayout static_layout(const rheo_config& c) {
     L.sum = take(2 * sizeof(float) * B * NP * P);
     L.table = take(sizeof(float) * B * NP * verify_table_width(c.K));
     L.rhat = take(sizeof(float) * B * NP * TL);
+    L.hdr = take(sizeof(int) * B * NP * 8);
+    L.child = take(sizeof(int) * B * NP * (c.K + 1) * 3);
+    L.tids = take(sizeof(int) * B * NP * TL);
+    L.tq = take(sizeof(float) * B * NP * TL);
+    L.cx = take(2 * sizeof(float) * B * NP * (c.K + 1));
+    L.tx = take(2 * sizeof(float) * B * NP * TL);
+    L.coin = take(sizeof(float) * B * NP * (c.K + 2));
     L.total = o;
     return L;
 }
@@ -137,6 +146,14 @@ extern "C" int rheo_verify_static(const rheo_config* cfg, const void* logits, in
     a.status = reinterpret_cast<unsigned*>(base + L.status);
     a.seg_mu = reinterpret_cast<float*>(base + L.mu);
     a.seg_sum = reinterpret_cast<float*>(base + L.sum);
+    a.row_ticket = reinterpret_cast<unsigned*>(base + L.row_ticket);
+    a.rec_hdr = reinterpret_cast<int*>(base + L.hdr);
+    a.rec_child = reinterpret_cast<int*>(base + L.child);
+    a.rec_tids = reinterpret_cast<int*>(base + L.tids);
+    a.rec_tq = reinterpret_cast<float*>(base + L.tq);
+    a.rec_cx = reinterpret_cast<float*>(base + L.cx);
+    a.rec_tx = reinterpret_cast<float*>(base + L.tx);
+    a.rec_coin = reinterpret_cast<float*>(base + L.coin);
     a.table = reinterpret_cast<float*>(base + L.table);
     a.rhat_tail = reinterpret_cast<float*>(base + L.rhat);
     a.res_best = reinterpret_cast<unsigned long long*>(base + L.best);

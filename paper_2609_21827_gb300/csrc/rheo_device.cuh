@@ -6,6 +6,7 @@
 // so a warp's load instruction covers 512 contiguous bytes.
 #pragma once
 
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -162,6 +163,13 @@ template <> struct Vec<1> {
         const float a3 = fast_exp2(fmaf(bf_lo(v.w), c, -mc)) + fast_exp2(fmaf(bf_hi(v.w), c, -mc));
         return (a0 + a1) + (a2 + a3);
     }
+    // bit i set when element i is >= t (t2: t as a bf16 pair; false for NaN)
+    __device__ static __forceinline__ uint32_t ge_bits(const uint4& v, uint32_t t2) {
+        const __nv_bfloat162 t = *reinterpret_cast<const __nv_bfloat162*>(&t2);
+        auto mk = [&](uint32_t w) { return __hge2_mask(*reinterpret_cast<const __nv_bfloat162*>(&w), t) & 0x00010001u; };
+        const uint32_t x = mk(v.x) | (mk(v.y) << 2) | (mk(v.z) << 4) | (mk(v.w) << 6);
+        return (x & 0x55u) | ((x >> 15) & 0xAAu);
+    }
     // elements [nv, 8) become -inf
     __device__ static __forceinline__ uint4 mask(uint4 v, int nv) {
         auto m = [](uint32_t w, int lo_idx, int nv) -> uint32_t {
@@ -181,6 +189,11 @@ template <> struct Vec<0> {
         const float a0 = fast_exp2(fmaf(__uint_as_float(v.x), c, -mc)) + fast_exp2(fmaf(__uint_as_float(v.y), c, -mc));
         const float a1 = fast_exp2(fmaf(__uint_as_float(v.z), c, -mc)) + fast_exp2(fmaf(__uint_as_float(v.w), c, -mc));
         return a0 + a1;
+    }
+    __device__ static __forceinline__ uint32_t ge_bits(const uint4& v, uint32_t t2) {
+        const float t = __uint_as_float(t2);
+        return (__uint_as_float(v.x) >= t ? 1u : 0u) | (__uint_as_float(v.y) >= t ? 2u : 0u) |
+               (__uint_as_float(v.z) >= t ? 4u : 0u) | (__uint_as_float(v.w) >= t ? 8u : 0u);
     }
     __device__ static __forceinline__ uint4 mask(uint4 v, int nv) {
         const uint32_t ni = 0xFF800000u;

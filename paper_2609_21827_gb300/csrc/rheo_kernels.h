@@ -81,6 +81,14 @@ struct VerifyArgs {
     unsigned* status;
     float* seg_mu;                  // [B*(N+1)*chunks]
     float* seg_sum;                 // [B*(N+1)*chunks*2] float-float partition sums
+    unsigned* row_ticket;           // [B*(N+1)] segments of the row streamed so far
+    int* rec_hdr;                   // [B*(N+1)*8] row records (see verify.cu)
+    int* rec_child;                 // [B*(N+1)*(K+1)*3]
+    int* rec_tids;                  // [B*(N+1)*TL]
+    float* rec_tq;                  // [B*(N+1)*TL]
+    float* rec_cx;                  // [B*(N+1)*(K+1)*2]
+    float* rec_tx;                  // [B*(N+1)*TL*2]
+    float* rec_coin;                // [B*(N+1)*(K+2)]
     float* table;                   // [B*(N+1)*table_width(K)] decision tables
     float* rhat_tail;               // [B*(N+1)*TL]
     unsigned long long* res_best;   // [B*3]

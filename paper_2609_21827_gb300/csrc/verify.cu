@@ -1,20 +1,19 @@
 // verify.cu -- RheoVerification (Algorithm 1) applied layer by layer (Theorem 1).
 //
-// Three launches on the caller's stream:
+// Two launches on the caller's stream:
 //
 // verify_stream_kernel: every warp streams its own contiguous run of 2 KB
 // chunks of the B*(N+1) target rows (16-byte loads straight into registers,
 // the next chunk in flight while the current one is summed), keeping a running
 // (max, sum exp((l - max) / T)) per lane.  Where a row segment of its run ends
-// the warp reduces that state and writes the segment's partial.  The warps
-// never wait for one another.
-//
-// verify_rows_kernel: one warp per pruned row builds the row's decision table:
-// lse_T from the partials, p at the surviving children and -- when the row's
-// sampled child survived -- r^ = max(0, p - q~) over the tail that child was
-// drawn from, the residual mass M = 1 - sum_tail min(p, q~), r^ at the
-// children, the Philox coins of the node, and the verdict of Algorithm 1 at
-// the node.  A row's verdict depends on nothing but the row itself.
+// the warp reduces that state and writes the segment's partial; the warp that
+// ends a row's last segment (arrival counter, never a wait) builds the row's
+// decision table: lse_T from the partials, p at the surviving children and --
+// when the row's sampled child survived -- r^ = max(0, p - q~) over the tail
+// that child was drawn from, the residual mass M = 1 - sum_tail min(p, q~), r^
+// at the children, the Philox coins of the node, and the verdict of Algorithm
+// 1 at the node.  A row's verdict depends on nothing but the row itself.  The
+// warps never wait for one another.
 //
 // residual_kernel, grid (chunks, B): each CTA stages its request's verdicts,
 // replays the walk from the root (a few comparisons per level), and takes part
@@ -41,12 +40,9 @@ __host__ __device__ __forceinline__ int table_width(int K) { return kTabP + 2 * 
 
 constexpr int kCV = 4;                     // 16-byte vectors per lane per chunk
 constexpr int kChunkBytesW = 32 * kCV * 16;  // bytes one warp takes per step
-constexpr int kRowWarps = 4;               // warps (rows) per CTA of the rows kernel
 
 struct WarpRow {
-    int32_t tok[kMaxSupport];   // children tokens
-    int32_t cgen[kMaxSupport];  // children gen ids
-    int32_t tids[kMaxSupport];  // tail ids
+    int32_t tok[kMaxSupport];   // children slots
     float pc[kMaxSupport];      // p at the children
     float rc[kMaxSupport];      // r^ at the children
     float pt[kMaxSupport];      // r^ over the tail
@@ -115,9 +111,241 @@ __device__ __forceinline__ void load_chunk(uint4 (&v)[kCV], const char* row, int
 
 }  // namespace
 
+// Row records, built by verify_prep_kernel from the trees while the stream
+// runs, so that a decision table needs two memory round trips (the record with
+// the partials, then the gathers from the target row):
+//   hdr[8]     n_child, first_child, sampled_child, gen id, q~(sampled child) bits
+//   child[3]   per surviving child: token, tail position (-1: off the tail), slot
+//   tids, tq   the tail list of the node's expansion (when its sampled child survived)
+//   cx, tx     l / T as float-float at the children and at the tail tokens
+//   coin       the node's K+2 Philox coins
+constexpr int kHdr = 8;
+
+// One warp per pruned row: the row's record.
+template <int DT>
+__global__ void __launch_bounds__(kThreads) verify_prep_kernel(const VerifyArgs a) {
+    using E = Elem<DT>;
+    grid_dependency_begin();
+    const Dims& n = a.n;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int K = n.K, TL = n.TL, NP = n.N + 1, m = n.m;
+    const int64_t r = (int64_t)blockIdx.x * kWarps + warp;
+    if (r >= (int64_t)n.B * NP) return;
+    const int b = (int)(r / NP);
+    const int64_t pb = (int64_t)b * NP, nb = (int64_t)b * n.G1;
+    int nc = a.pr.n_child[r], fc = a.pr.first_child[r], sc = a.pr.sampled_child[r];
+    if (!pruned_row_ok(nc, fc, sc, K, n.N)) {
+        if (lane == 0) atomicOr(a.status, kStInternal);
+        nc = 0;
+        sc = -1;
+    }
+    const int gen = a.pr.gen_id[r];
+    int* hdr = a.rec_hdr + r * kHdr;
+    int* child = a.rec_child + r * (K + 1) * 3;
+    // children: token, gen id (slot), and the sampled child's token
+    int ctok[4], cslot[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int i = lane + 32 * q;
+        ctok[q] = (i < nc) ? a.pr.token[pb + fc + i] : -1;
+        cslot[q] = (i < nc) ? slot_of(K, min(max(a.pr.gen_id[pb + fc + i], 1), (int)n.G1 - 1)) : 0;
+    }
+    const int ytok = (sc >= 0) ? a.pr.token[pb + sc] : -1;
+    const int ygen = (sc >= 0) ? a.pr.gen_id[pb + sc] : 1;
+    float qs = 0.0f;
+    int ypos = -1;
+    if (sc >= 0) {
+        qs = a.tree.qtilde[nb + min(max(ygen, 1), (int)n.G1 - 1)];
+        const int64_t e = expansion_of_child(K, ygen, n.G1, n.E);
+        const int64_t q0 = ((int64_t)b * n.E + e) * TL;
+        for (int i0 = 0; i0 < TL; i0 += 32) {
+            const int i = i0 + lane;
+            int tok = -1;
+            if (i < TL) {
+                tok = a.tree.tail_ids[q0 + i];
+                a.rec_tids[r * TL + i] = tok;
+                a.rec_tq[r * TL + i] = a.tree.tail_q[q0 + i];
+            }
+            const unsigned hit = __ballot_sync(0xFFFFFFFFu, i < TL && tok == ytok);
+            if (hit && ypos < 0) ypos = i0 + __ffs(hit) - 1;
+        }
+    }
+    __syncwarp();  // the copied tail is read back below
+    // tail positions: the sampled child at ypos, fills at the next ranks with
+    // ypos skipped, leads off the tail; anything else is searched for
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int i = lane + 32 * q;
+        if (i >= nc) continue;
+        int pos = -1;
+        if (sc >= 0) {
+            const int j = cslot[q], qf = j - m - 1;
+            pos = (j < m) ? -1 : (j == m) ? ypos : qf + (qf >= ypos ? 1 : 0);
+            if (pos >= TL || (pos >= 0 && a.rec_tids[r * TL + pos] != ctok[q]) || (pos < 0 && j >= m)) {
+                pos = -1;
+                for (int t = 0; t < TL; ++t)
+                    if (a.rec_tids[r * TL + t] == ctok[q]) pos = t;
+            }
+        }
+        child[3 * i + 0] = ctok[q];
+        child[3 * i + 1] = pos;
+        child[3 * i + 2] = cslot[q];
+    }
+    // target logits at the children and at the tail, as l / T
+    const float T = a.T[b];
+    const char* row = a.logits + r * a.row_stride_bytes;
+    auto scaled = [&](int tok) -> FF {
+        const float l = (tok >= 0 && tok < n.V) ? E::value(E::load_scalar(row, tok)) : -INFINITY;
+        return ff_div(l, T);
+    };
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int i = lane + 32 * q;
+        if (i < nc) {
+            const FF x = scaled(ctok[q]);
+            a.rec_cx[2 * (r * (K + 1) + i)] = x.hi;
+            a.rec_cx[2 * (r * (K + 1) + i) + 1] = x.lo;
+        }
+        if (sc >= 0 && i < TL) {
+            const FF x = scaled(a.rec_tids[r * TL + i]);
+            a.rec_tx[2 * (r * TL + i)] = x.hi;
+            a.rec_tx[2 * (r * TL + i) + 1] = x.lo;
+        }
+    }
+    const uint64_t seed = a.seed[b], off = a.offset[b];
+    for (int i = lane; i < K + 2; i += 32) a.rec_coin[r * (K + 2) + i] = uniform(seed, off, kTagVerify, gen, (uint64_t)i);
+    if (lane == 0) {
+        hdr[0] = nc;
+        hdr[1] = fc;
+        hdr[2] = sc;
+        hdr[3] = gen;
+        hdr[4] = __float_as_int(qs);
+    }
+}
+
+// exp(x - c) for x = l / T and c as float-float (the arithmetic of exp_scaled_minus)
+__device__ __forceinline__ float exp_ff_minus(FF x, FF c) {
+    if (!(x.hi > -INFINITY && x.hi < INFINITY)) return expf(x.hi - c.hi);
+    return expf(__fsub_rn(x.hi, c.hi) + (x.lo - c.lo));
+}
+
+// The decision table of pruned row r (Algorithm 1 at the node), built by one
+// warp from the row's segment partials and its record.
+template <int DT>
+__device__ __noinline__ void finalize_row(const VerifyArgs& a, int64_t r, WarpRow& w) {
+    const Dims& n = a.n;
+    const int lane = threadIdx.x & 31;
+    const int K = n.K, TL = n.TL, NP = n.N + 1;
+    const int b = (int)(r / NP);
+    const int cpr = n.chunks;
+    const int TW = table_width(K);
+    const TileSplit sp{(int64_t)n.B * NP * cpr, a.units};
+    const int nseg = sp.owner(r * cpr + cpr - 1) - sp.owner(r * cpr) + 1;
+    // round trip 1: the record and the partials
+    const int* hdr = a.rec_hdr + r * kHdr;
+    const int* child = a.rec_child + r * (K + 1) * 3;
+    const int nc = __ldcg(hdr + 0), fc = __ldcg(hdr + 1), sc = __ldcg(hdr + 2);
+    const float qs = __int_as_float(__ldcg(hdr + 4));
+    int cpos[4], cslot[4];
+    float tq[4];
+    FF cx[4], tx[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int i = lane + 32 * q;
+        const bool c_ok = i < K + 1, t_ok = i < TL;
+        cpos[q] = c_ok ? __ldcg(child + 3 * i + 1) : -1;
+        cslot[q] = c_ok ? __ldcg(child + 3 * i + 2) : 0;
+        cx[q] = c_ok ? FF{__ldcg(a.rec_cx + 2 * (r * (K + 1) + i)), __ldcg(a.rec_cx + 2 * (r * (K + 1) + i) + 1)}
+                     : FF{-INFINITY, 0.0f};
+        tq[q] = t_ok ? __ldcg(a.rec_tq + r * TL + i) : 0.0f;
+        tx[q] = t_ok ? FF{__ldcg(a.rec_tx + 2 * (r * TL + i)), __ldcg(a.rec_tx + 2 * (r * TL + i) + 1)}
+                     : FF{-INFINITY, 0.0f};
+    }
+    const float coin_l = (lane < K + 2) ? __ldcg(a.rec_coin + r * (K + 2) + lane) : 0.0f;
+    const float T = a.T[b];
+    const FF lse = combine_lse(a.seg_mu + r * cpr, a.seg_sum + 2 * r * cpr, nseg, T);
+    float* tab = a.table + r * TW;
+    if (lane == 0) {
+        tab[3] = lse.hi;
+        tab[4] = lse.lo;
+        if (a.row_lse) a.row_lse[r] = __fadd_rn(lse.hi, lse.lo);
+        if (!(lse.hi > -INFINITY)) atomicOr(a.status, kStEmptyRow);
+        if ((r % NP) == 0 && (!(T > 0.0f) || isinf(T))) atomicOr(a.status, kStBadTemperature);
+    }
+    // r^ over the tail and the overlap sum of min(p, q~) (sampled child survived)
+    FF ov{0.0f, 0.0f};
+    if (sc >= 0) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int i = lane + 32 * q;
+            if (i >= TL) continue;
+            const float pt = exp_ff_minus(tx[q], lse);
+            const float d = __fsub_rn(pt, tq[q]);
+            const float rh = d > 0.0f ? d : 0.0f;
+            w.pt[i] = rh;
+            a.rhat_tail[r * TL + i] = rh;
+            ov = ff_add(ov, fminf(pt, tq[q]));
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) ov = ff_add(ov, ff_shfl_xor(ov, o));
+    for (int i = lane; i < K + 2; i += 32) {
+        const float u = (i == lane) ? coin_l : __ldcg(a.rec_coin + r * (K + 2) + i);
+        w.coin[i] = u;
+        tab[kTabP + 2 * (K + 1) + i] = u;
+    }
+    __syncwarp();
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int i = lane + 32 * q;
+        if (i >= nc) continue;
+        const float p = exp_ff_minus(cx[q], lse);
+        const float rh = (sc >= 0 && cpos[q] >= 0 && cpos[q] < TL) ? w.pt[cpos[q]] : p;
+        w.pc[i] = p;
+        w.rc[i] = rh;
+        w.tok[i] = cslot[q];  // the slot decides the coin
+        tab[kTabP + i] = p;
+        tab[kTabP + (K + 1) + i] = rh;
+    }
+    __syncwarp();
+    if (lane == 0) {
+        // Algorithm 1 at this node: stochastic first, then recursive rejection in slot order
+        FF M{1.0f, 0.0f};
+        int acc = -1, use_tail = 0;
+        if (sc >= 0) {
+            if (__fmul_rn(w.coin[0], qs) <= w.pc[sc - fc]) {
+                acc = sc;
+            } else {
+                M = ff_add(FF{1.0f, 0.0f}, ff_neg(ov));
+                use_tail = 1;
+            }
+        }
+        const FF M0 = M;
+        if (acc < 0)
+            for (int c2 = 0; c2 < nc; ++c2) {
+                if (fc + c2 == sc) continue;
+                const float eta = w.coin[1 + w.tok[c2]];
+                const float rv = use_tail ? w.rc[c2] : w.pc[c2];
+                if (ff_le(ff_mul(eta, M), rv)) {  // eta * M <= r^(u_i)
+                    acc = fc + c2;
+                    break;
+                }
+                M = ff_add(M, -rv);
+            }
+        tab[0] = M0.hi;
+        tab[1] = M0.lo;
+        tab[2] = qs;
+        tab[5] = (float)use_tail;
+        tab[6] = (float)acc;
+    }
+}
+
 template <int DT, bool ALIGNED>
 __global__ void __launch_bounds__(kThreads, 2) verify_stream_kernel(const VerifyArgs a) {
-    grid_dependency_begin();
+    // streaming needs nothing from the grids before this one: let the next grid
+    // launch now, and wait for the row records only before the first table
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    __shared__ WarpRow wrs[kWarps];
     using E = Elem<DT>;
     using W = Vec<DT>;
     constexpr int VEC = E::VEC;
@@ -170,146 +398,29 @@ __global__ void __launch_bounds__(kThreads, 2) verify_stream_kernel(const Verify
         // ---- end of this warp's segment of row r: its partial ------------------
         float M;
         const FF Sw = warp_partition(mu, sum, c, M);
+        int last = 0;
         if (lane == 0) {
-            const int seg = u - sp.owner(r * cpr);
+            const int first = sp.owner(r * cpr);
+            const int seg = u - first;
+            const int nseg = sp.owner(r * cpr + cpr - 1) - first + 1;
             a.seg_mu[r * cpr + seg] = M;
             a.seg_sum[2 * (r * cpr + seg)] = Sw.hi;
             a.seg_sum[2 * (r * cpr + seg) + 1] = Sw.lo;
             if (isnan(Sw.hi) || M == INFINITY) atomicOr(a.status, kStBadLogit);
+            // the warp that ends the row's last segment builds its decision table
+            __threadfence();
+            last = (atomicAdd(a.row_ticket + r, 1u) == (unsigned)nseg - 1u) ? 1 : 0;
+            if (last) {
+                a.row_ticket[r] = 0u;  // ready for the next call
+                __threadfence();
+            }
+        }
+        if (__shfl_sync(0xFFFFFFFFu, last, 0)) {
+            asm volatile("griddepcontrol.wait;" ::: "memory");
+            finalize_row<DT>(a, r, wrs[warp]);
         }
         mu = -INFINITY;
         sum = 0.0f;
-    }
-}
-
-// One warp per pruned row: the row's decision table (Algorithm 1 at the node).
-template <int DT>
-__global__ void __launch_bounds__(32 * kRowWarps) verify_rows_kernel(const VerifyArgs a) {
-    grid_dependency_begin();
-    using E = Elem<DT>;
-    __shared__ WarpRow wrs[kRowWarps];
-    const Dims& n = a.n;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int V = n.V, K = n.K, TL = n.TL, NP = n.N + 1;
-    const int64_t r = (int64_t)blockIdx.x * kRowWarps + warp;
-    if (r >= (int64_t)n.B * NP) return;
-    WarpRow& w = wrs[warp];
-    const int b = (int)(r / NP);
-    const int cpr = n.chunks;
-    const int TW = table_width(K);
-    const TileSplit sp{(int64_t)n.B * NP * cpr, a.units};
-    const int nseg = sp.owner(r * cpr + cpr - 1) - sp.owner(r * cpr) + 1;
-    const float T = a.T[b];
-    int nc = a.pr.n_child[r], fc = a.pr.first_child[r], sc = a.pr.sampled_child[r];
-    const int gen = a.pr.gen_id[r];
-    const FF lse = combine_lse(a.seg_mu + r * cpr, a.seg_sum + 2 * r * cpr, nseg, T);
-    float* tab = a.table + r * TW;
-
-    if (!pruned_row_ok(nc, fc, sc, K, n.N)) {
-        if (lane == 0) atomicOr(a.status, kStInternal);
-        nc = 0;
-        sc = -1;
-    }
-    if (lane == 0) {
-        tab[3] = lse.hi;
-        tab[4] = lse.lo;
-        if (a.row_lse) a.row_lse[r] = __fadd_rn(lse.hi, lse.lo);
-        if (!(lse.hi > -INFINITY)) atomicOr(a.status, kStEmptyRow);
-        if ((r % NP) == 0 && (!(T > 0.0f) || isinf(T))) atomicOr(a.status, kStBadTemperature);
-    }
-    const int64_t pb = (int64_t)b * NP;
-    const int64_t e = (sc >= 0) ? expansion_of_child(K, a.pr.gen_id[pb + sc], n.G1, n.E) : 0;
-    const int64_t q0 = ((int64_t)b * n.E + e) * TL;
-    const char* row = a.logits + r * a.row_stride_bytes;
-    auto logit = [&](int tok) -> float { return (tok >= 0 && tok < V) ? E::value(E::load_scalar(row, tok)) : -INFINITY; };
-
-    for (int i = lane; i < nc; i += 32) {
-        const int tok = a.pr.token[pb + fc + i];
-        w.tok[i] = tok;
-        w.cgen[i] = a.pr.gen_id[pb + fc + i];
-        w.pc[i] = exp_scaled_minus(logit(tok), T, lse);
-    }
-    // the tail of the sampled child's draw, when that child survived
-    FF ov{0.0f, 0.0f};
-    if (sc >= 0)
-        for (int i = lane; i < TL; i += 32) {
-            const int tok = a.tree.tail_ids[q0 + i];
-            const float qi = a.tree.tail_q[q0 + i];
-            const float pt = exp_scaled_minus(logit(tok), T, lse);
-            const float d = __fsub_rn(pt, qi);
-            const float rh = d > 0.0f ? d : 0.0f;
-            w.tids[i] = tok;
-            w.pt[i] = rh;
-            a.rhat_tail[r * TL + i] = rh;
-            ov = ff_add(ov, fminf(pt, qi));
-        }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) ov = ff_add(ov, ff_shfl_xor(ov, o));
-    const uint64_t seed = a.seed[b], off = a.offset[b];
-    for (int i = lane; i < K + 2; i += 32) {
-        const float u = uniform(seed, off, kTagVerify, gen, (uint64_t)i);
-        w.coin[i] = u;
-        tab[kTabP + 2 * (K + 1) + i] = u;
-    }
-    __syncwarp();
-    // tail position of the sampled child: fills sit at the next ranks, Y skipped
-    int ypos = -1;
-    if (sc >= 0) {
-        const int ytok = w.tok[sc - fc];
-        for (int i0 = 0; i0 < TL && ypos < 0; i0 += 32) {
-            const unsigned hit = __ballot_sync(0xFFFFFFFFu, i0 + lane < TL && w.tids[i0 + lane] == ytok);
-            if (hit) ypos = i0 + __ffs(hit) - 1;
-        }
-    }
-    for (int i = lane; i < nc; i += 32) {
-        int pos = -1;
-        if (sc >= 0) {
-            const int j = slot_of(K, w.cgen[i]);
-            const int qf = j - n.m - 1;
-            pos = (j < n.m) ? -1 : (j == n.m) ? ypos : qf + (qf >= ypos ? 1 : 0);
-            if (pos >= TL || (pos >= 0 && w.tids[pos] != w.tok[i]) || (pos < 0 && j >= n.m)) {
-                pos = -1;  // not the layout of the expansion: search the tail
-                for (int q = 0; q < TL; ++q)
-                    if (w.tids[q] == w.tok[i]) pos = q;
-            }
-        }
-        const float p = w.pc[i];
-        const float rh = (pos >= 0) ? w.pt[pos] : p;
-        w.rc[i] = rh;
-        tab[kTabP + i] = p;
-        tab[kTabP + (K + 1) + i] = rh;
-    }
-    __syncwarp();
-    if (lane == 0) {
-        // Algorithm 1 at this node: stochastic first, then recursive rejection in slot order
-        const float qs = (sc >= 0) ? a.tree.qtilde[(int64_t)b * n.G1 + w.cgen[sc - fc]] : 0.0f;
-        FF M{1.0f, 0.0f};
-        int acc = -1, use_tail = 0;
-        if (sc >= 0) {
-            if (__fmul_rn(w.coin[0], qs) <= w.pc[sc - fc]) {
-                acc = sc;
-            } else {
-                M = ff_add(FF{1.0f, 0.0f}, ff_neg(ov));
-                use_tail = 1;
-            }
-        }
-        const FF M0 = M;
-        if (acc < 0)
-            for (int c2 = 0; c2 < nc; ++c2) {
-                if (fc + c2 == sc) continue;
-                const float eta = w.coin[1 + slot_of(K, w.cgen[c2])];
-                const float rv = use_tail ? w.rc[c2] : w.pc[c2];
-                if (ff_le(ff_mul(eta, M), rv)) {  // eta * M <= r^(u_i)
-                    acc = fc + c2;
-                    break;
-                }
-                M = ff_add(M, -rv);
-            }
-        tab[0] = M0.hi;
-        tab[1] = M0.lo;
-        tab[2] = qs;
-        tab[5] = (float)use_tail;
-        tab[6] = (float)acc;
     }
 }
 
@@ -324,7 +435,7 @@ __device__ __forceinline__ unsigned long long pack_key(float key, int64_t id) {
     return ((unsigned long long)ord_f32(key) << 32) | (0xFFFFFFFFu - (uint32_t)id);
 }
 
-template <int DT>
+template <int DT, bool ALIGNED>
 __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) {
     grid_dependency_begin();
     using E = Elem<DT>;
@@ -384,26 +495,23 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     const float lse = __ldcg(tu + 3);
     const float T = a.T[b];
     const uint64_t seed = a.seed[b], off = a.offset[b];
-    const int gen_u = a.pr.gen_id[rowg];
-    const int nc = a.pr.n_child[rowg], fc = a.pr.first_child[rowg];
-    const int nc_ok = (nc >= 0 && nc <= K + 1 && fc >= 0 && fc + nc <= NP) ? nc : 0;
-    int64_t e = 0;
-    if (use_tail) {
-        const int sc = a.pr.sampled_child[rowg];
-        e = expansion_of_child(K, (sc >= 0 && sc < NP) ? a.pr.gen_id[pb + sc] : 1, n.G1, n.E);
-    }
-    const int32_t* tids = a.tree.tail_ids + ((int64_t)b * n.E + e) * TL;
+    // the stopping row's record: children and (after a rejection) its tail
+    const int* hdr = a.rec_hdr + rowg * kHdr;
+    const int nc = __ldcg(hdr + 0), gen_u = __ldcg(hdr + 3);
+    const int nc_ok = (nc >= 0 && nc <= K + 1) ? nc : 0;
+    const int* rchild = a.rec_child + rowg * (K + 1) * 3;
+    const int32_t* tids = a.rec_tids + rowg * TL;
     const char* row = a.logits + rowg * a.row_stride_bytes;
     const int64_t e_lo = (int64_t)k * kResChunk;
 
     for (int c = tid; c < nc_ok; c += kThreads) {
-        const int tok = a.pr.token[pb + fc + c];
+        const int tok = __ldcg(rchild + 3 * c);
         if (tok >= e_lo && tok < e_lo + kResChunk)
             atomicOr(&excl_bits[(tok - e_lo) >> 5], 1u << ((tok - e_lo) & 31));
     }
     if (use_tail)
         for (int i = tid; i < TL; i += kThreads) {
-            const int tok = tids[i];
+            const int tok = __ldcg(tids + i);
             if (tok >= e_lo && tok < e_lo + kResChunk)
                 atomicOr(&tail_bits[(tok - e_lo) >> 5], 1u << ((tok - e_lo) & 31));
         }
@@ -414,6 +522,9 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     unsigned long long best = 0ull;
     {
         const int64_t e0 = e_lo + (int64_t)tid * kResPer;
+        uint4 xv[kResPer / E::VEC];  // this thread's elements of the stopping row
+#pragma unroll
+        for (int j = 0; j < kResPer / E::VEC; ++j) xv[j] = load_vec<DT, ALIGNED>(row, e0 + j * E::VEC, V);
 #pragma unroll
         for (int h = 0; h < kResPer / 4; ++h) {
             if (e0 + 4 * h >= V) break;
@@ -424,7 +535,8 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
                 if (id >= V) break;
                 const int li = (int)(id - e_lo);
                 if (((excl_bits[li >> 5] | tail_bits[li >> 5]) >> (li & 31)) & 1u) continue;
-                const float x = E::value(E::load_scalar(row, id));
+                const int q = 4 * h + i;
+                const float x = E::value(E::raw(xv[q / E::VEC], q % E::VEC));
                 const float g = gumbel(u01(word_of(rnd, i)));
                 const float key = __fadd_rn(__fsub_rn(__fdiv_rn(x, T), lse), g);
                 if (key > -INFINITY) {
@@ -437,7 +549,7 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     // tail entries use log r^ (zero mass after a rejection: no key)
     if (use_tail)
         for (int i = tid; i < TL; i += kThreads) {
-            const int tok = tids[i];
+            const int tok = __ldcg(tids + i);
             if (tok < e_lo || tok >= e_lo + kResChunk) continue;
             const int li = tok - (int)e_lo;
             if ((excl_bits[li >> 5] >> (li & 31)) & 1u) continue;
@@ -462,7 +574,7 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
         unsigned long long b1 = 0ull, b2 = 0ull;
         for (int64_t id = tid; id < V; id += kThreads) {
             bool ex = false;
-            for (int c = 0; c < nc_ok; ++c) ex |= (a.pr.token[pb + fc + c] == id);
+            for (int c = 0; c < nc_ok; ++c) ex |= (__ldcg(rchild + 3 * c) == id);
             const float x = E::value(E::load_scalar(row, id));
             const float g = gumbel(uniform(seed, off, kTagResidual, gen_u, (uint64_t)id));
             const float key = __fadd_rn(__fdiv_rn(x, T), g);
@@ -484,6 +596,11 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
 }
 
 cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid, cudaStream_t s) {
+    const int64_t rows = (int64_t)a.n.B * (a.n.N + 1);
+    const dim3 gp((unsigned)((rows + kWarps - 1) / kWarps));
+    cudaError_t e0 = (dtype == 1) ? launch_dependent(verify_prep_kernel<1>, gp, dim3(kThreads), 0, s, a)
+                                  : launch_dependent(verify_prep_kernel<0>, gp, dim3(kThreads), 0, s, a);
+    if (e0 != cudaSuccess) return e0;
     auto go_stream = [&](auto kern) {
         return launch_dependent(kern, dim3(grid), dim3(kThreads), 0, s, a);
     };
@@ -491,14 +608,12 @@ cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid
     if (dtype == 1) err = aligned ? go_stream(verify_stream_kernel<1, true>) : go_stream(verify_stream_kernel<1, false>);
     else err = aligned ? go_stream(verify_stream_kernel<0, true>) : go_stream(verify_stream_kernel<0, false>);
     if (err != cudaSuccess) return err;
-    const int64_t rows = (int64_t)a.n.B * (a.n.N + 1);
-    const int g1 = (int)((rows + kRowWarps - 1) / kRowWarps);
-    err = (dtype == 1) ? launch_dependent(verify_rows_kernel<1>, dim3(g1), dim3(32 * kRowWarps), 0, s, a)
-                       : launch_dependent(verify_rows_kernel<0>, dim3(g1), dim3(32 * kRowWarps), 0, s, a);
-    if (err != cudaSuccess) return err;
     const dim3 g2((a.n.V + kResChunk - 1) / kResChunk, a.n.B);
-    return (dtype == 1) ? launch_dependent(residual_kernel<1>, g2, dim3(kThreads), 0, s, a)
-                        : launch_dependent(residual_kernel<0>, g2, dim3(kThreads), 0, s, a);
+    if (dtype == 1)
+        return aligned ? launch_dependent(residual_kernel<1, true>, g2, dim3(kThreads), 0, s, a)
+                       : launch_dependent(residual_kernel<1, false>, g2, dim3(kThreads), 0, s, a);
+    return aligned ? launch_dependent(residual_kernel<0, true>, g2, dim3(kThreads), 0, s, a)
+                   : launch_dependent(residual_kernel<0, false>, g2, dim3(kThreads), 0, s, a);
 }
 
 int verify_table_width(int K) { return table_width(K); }

@@ -51,6 +51,7 @@ struct E2Smem {
 
 struct HistSel {
     int bin, cbin, above, tie_n;
+    int cbefore[kCoarseBins];  // keys in coarse bins above each coarse bin
 };
 
 __device__ __forceinline__ unsigned long long make_key(uint32_t k32, int64_t id) {
@@ -185,6 +186,7 @@ __device__ void hist_boundary(const unsigned* coarse, const unsigned* fine, int 
     const int c = (int)coarse[cb];
     int total;
     const int before = red_scan(c, total, red, par);
+    hs.cbefore[cb] = before;
     if (tid == 0) {
         hs.bin = -1;
         hs.tie_n = 0;
@@ -208,7 +210,11 @@ __device__ void hist_boundary(const unsigned* coarse, const unsigned* fine, int 
             const int t2 = __shfl_sync(0xFFFFFFFFu, inc, 31);
             if (acc + t2 >= k) {
                 const int L2 = __ffs(__ballot_sync(0xFFFFFFFFu, acc + inc >= k)) - 1;
-                if (lane == 0) hs.bin = f0 - L2;
+                const int above = acc + __shfl_sync(0xFFFFFFFFu, inc - w, L2);
+                if (lane == 0) {
+                    hs.bin = f0 - L2;
+                    hs.above = above;  // keys in higher fine bins
+                }
                 break;
             }
             acc += t2;
@@ -217,21 +223,64 @@ __device__ void hist_boundary(const unsigned* coarse, const unsigned* fine, int 
     __syncthreads();
 }
 
-// Append the keys x with fine bin >= bin among xs[0, cnt) (this warp's keys) to
-// tmp at positions from hs.tie_n, one shared atomic per 32 keys.
-__device__ __forceinline__ void warp_gather_from(const unsigned long long* xs, int cnt, int bin,
-                                                 unsigned long long* tmp, int cap, HistSel& hs) {
-    const int lane = threadIdx.x & 31;
-    for (int j0 = 0; j0 < cnt; j0 += 32) {
-        const unsigned long long x = (j0 + lane < cnt) ? xs[j0 + lane] : 0ull;
-        const bool take = x != 0ull && (int)(x >> kFineShift) >= bin;
-        const unsigned bal = __ballot_sync(0xFFFFFFFFu, take);
-        int base = 0;
-        if (lane == 0 && bal) base = atomicAdd(&hs.tie_n, __popc(bal));
-        base = __shfl_sync(0xFFFFFFFFu, base, 0);
-        const int pos = base + __popc(bal & ((1u << lane) - 1u));
-        if (take && pos < cap) tmp[pos] = x;
+// The k best keys in descending order into sorted[0, k), by a counting sort on
+// the fine histogram (after hist_boundary): every fine bin from the boundary bin
+// up gets its offset (keys in higher bins) in place of its count, the keys of
+// those bins are scattered (scatter(f): f(x) for each such key, called by all
+// threads) into tmp in bin order, and each is ranked among the keys of its own
+// bin.  Returns min(k, keys at or above the boundary).  The fine histogram is
+// consumed.
+template <class Scatter, class CoarseCount>
+__device__ int hist_sort_top(Scatter scatter, CoarseCount coarse_count, int k, unsigned* fine,
+                             unsigned long long* tmp, unsigned long long* sorted, HistSel& hs) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int bstar = hs.bin < 0 ? 0 : hs.bin;
+    const int cstar = bstar / kFinePerCoarse;
+    {
+        // each warp converts the non-empty coarse bins of its lanes (lane t: coarse
+        // bin 255 - t), the 64 fine bins two per lane with a warp scan, from the top
+        static_assert(kFinePerCoarse == 64, "two fine bins per lane");
+        const int cbl = kCoarseBins - 1 - tid;
+        unsigned todo = __ballot_sync(0xFFFFFFFFu, cbl >= cstar && coarse_count(cbl) > 0);
+        while (todo) {
+            const int L = __ffs(todo) - 1;
+            todo &= todo - 1u;
+            const int C = kCoarseBins - 1 - (warp * 32 + L);
+            const int f0 = C * kFinePerCoarse + kFinePerCoarse - 1 - 2 * lane, f1 = f0 - 1;
+            const int c0 = (int)fine[f0], c1 = (int)fine[f1];
+            int incl = c0 + c1;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+                if (lane >= o) incl += y;
+            }
+            const int o0 = hs.cbefore[C] + incl - c0 - c1;
+            fine[f0] = (unsigned)o0;
+            fine[f1] = (unsigned)(o0 + c0);
+            if (hs.bin >= 0 && f0 == bstar) hs.tie_n = o0 + c0;  // keys at or above the boundary bin
+            if (hs.bin >= 0 && f1 == bstar) hs.tie_n = o0 + c0 + c1;
+        }
+        if (hs.bin < 0 && tid == 0) hs.tie_n = hs.cbefore[0] + coarse_count(0);  // fewer than k: all keys
     }
+    __syncthreads();
+    const int nsel = hs.tie_n;
+    scatter([&](unsigned long long x) {
+        const int f = (int)(x >> kFineShift);
+        if (f >= bstar) tmp[atomicAdd(&fine[f], 1u)] = x;
+    });
+    __syncthreads();
+    const int kk = nsel < k ? nsel : k;
+    for (int p = tid; p < nsel; p += kThreads) {
+        const unsigned long long x = tmp[p];
+        const int f = (int)(x >> kFineShift);
+        const int start = (f % kFinePerCoarse == kFinePerCoarse - 1) ? hs.cbefore[f / kFinePerCoarse] : (int)fine[f + 1];
+        const int end = (int)fine[f];
+        int rank = start;
+        for (int q = start; q < end; ++q) rank += tmp[q] > x;
+        if (rank < kk) sorted[rank] = x;
+    }
+    __syncthreads();
+    return kk;
 }
 
 // Block-wide: append the keys with fine bin >= bin among get(i), i < n.
@@ -489,11 +538,13 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
         };
         // the k best: all keys at or above the fine bin of the k-th, ranked
         hist_boundary(coarse, fine, target, hs, red, par);
-        warp_gather_from(region, cnt, hs.bin < 0 ? 0 : hs.bin, tmpk, kTmpCap, hs);
-        __syncthreads();
         int written;
-        if (hs.tie_n <= kTmpCap) {
-            written = rank_gathered(tmpk, target, e2.sorted, hs);
+        if (hs.bin < 0 || hs.above + (int)fine[hs.bin] <= kTmpCap) {
+            written = hist_sort_top(
+                [&](auto put) {
+                    for (int j = lane; j < cnt; j += 32) put(region[j]);
+                },
+                [&](int c) { return coarse[c]; }, target, fine, tmpk, e2.sorted, hs);
         } else {  // a tie class too large for the list
             const unsigned long long thr = block_kth_key(rkey, kWarps * kRegion, target, s_hist, s_sel);
             if (tid == 0) hs.tie_n = 0;
@@ -543,11 +594,14 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
             __syncthreads();
             auto mkey = [&](int i) { return keys[i]; };
             hist_boundary(coarse, fine, S, hs, red, par);
-            block_gather_bin(mkey, nkeys, hs.bin < 0 ? 0 : hs.bin, tmpk, kTmpCap, hs);
-            __syncthreads();
             int got;
-            if (hs.tie_n <= kTmpCap) {
-                got = rank_gathered(tmpk, S, e2.sorted, hs);
+            if (hs.bin < 0 || hs.above + (int)fine[hs.bin] <= kTmpCap) {
+                got = hist_sort_top(
+                    [&](auto put) {
+                        for (int i = tid; i < nkeys; i += kThreads)
+                            if (keys[i]) put(keys[i]);
+                    },
+                    [&](int c) { return coarse[c]; }, S, fine, tmpk, e2.sorted, hs);
             } else {
                 const unsigned long long thr = block_kth_key(mkey, nkeys, S, s_hist, s_sel);
                 if (tid == 0) hs.tie_n = 0;

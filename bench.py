@@ -15,6 +15,7 @@ over ranks and value counts the tree-steps of all ranks.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -27,6 +28,34 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "tree-steps/sec (expand+prune+verify) at batch B, vocab V; HBM GB/s vs peak"
+
+
+KERNEL_SOURCES = ("expand.cu", "rheo_device.cuh", "rheo_kernels.h", "stream.cuh")
+
+
+def kernel_sources_sha() -> str:
+    """sha256 over the sources the expand kernel is compiled from (traffic taken
+    from an ncu capture is reported only while these are unchanged)."""
+    import hashlib
+
+    h = hashlib.sha256()
+    for name in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2609_21827_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def _traffic(key: str):
+    """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from
+    the committed ncu summary, or None if absent or taken on other sources."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            e = json.load(f).get(key)
+        if e and e.get("sources_sha256") == kernel_sources_sha():
+            return e["bytes_per_launch"]
+    except Exception:
+        pass
+    return None
 
 
 def _peaks():
@@ -236,6 +265,8 @@ def main(argv=None):
     ap.add_argument("--workload", default="qwen3_batch")
     ap.add_argument("--e2e-steps", type=int, default=50)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="override the workload's batch (a smaller case of the same kernels, for profiling)")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)
 
@@ -243,6 +274,8 @@ def main(argv=None):
     from paper_2609_21827_gb300 import synth
 
     w = synth.WORKLOADS[args.workload]
+    if args.batch > 0 and args.batch != w.batch:
+        w = dataclasses.replace(w, name=f"{w.name}_b{args.batch}", batch=args.batch)
     if args.impl == "reference":
         return run_reference(args, w)
 
@@ -395,14 +428,18 @@ def main(argv=None):
     exp_gbs = expand_bytes / (exp_ms / 1e3) / 1e9
     ver_gbs = verify_bytes / (ver_ms / 1e3) / 1e9
     step_gbs = (expand_bytes + verify_bytes) / (secs / args.steps) / 1e9
-    dominant = "expand" if exp_ms >= ver_ms else "verify"
-    ach = exp_gbs if dominant == "expand" else ver_gbs
-    traffic = None
-    try:
-        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
-            traffic = json.load(f).get(f"{w.name}:{dominant}")
-    except Exception:
-        pass
+    # the dominant kernel: expand_kernel at depths >= 2 (B*K frontier rows per
+    # launch, most of the step's time); algorithmic bytes = one read of its rows
+    if D >= 2:
+        dom_name = f"expand_kernel (depth >= 2, {w.batch * w.K} rows per launch)"
+        dom_bytes = w.batch * w.K * w.vocab * esz
+        dom_ms = sum(by_depth[1:]) / n_k / (D - 1)
+        dom_key = f"{w.name}:expand_d2"
+    else:
+        dom_name, dom_bytes, dom_ms, dom_key = f"expand_kernel (depth 1, {w.batch} rows)", \
+            w.batch * w.vocab * esz, by_depth[0] / n_k, f"{w.name}:expand_d1"
+    ach = dom_bytes / (dom_ms / 1e3) / 1e9
+    traffic = _traffic(dom_key)
     cpu = None if args.no_cpu_baseline else cpu_baseline(w, draft)
     line = {
         "metric": METRIC, "value": world * args.steps / secs, "unit": "tree-steps/s", "n_gpus": world,
@@ -413,14 +450,15 @@ def main(argv=None):
                    "bytes_per_step": expand_bytes + verify_bytes, "l2": "inputs 4x larger than L2, no flush",
                    "parallelism": f"replicas{world}", "cuda_graph": True,
                    "kernel_timing": "separate graph with event nodes" if graph_events else "eager steps"},
-        "roofline": {"bound": "hbm", "kernel": dominant, "achieved": ach, "peak": peak, "unit": "GB/s",
-                     "frac": ach / peak, "peak_kind": peak_kind, "traffic": traffic},
+        "roofline": {"bound": "hbm", "kernel": dom_name, "achieved": ach, "peak": peak, "unit": "GB/s",
+                     "frac": ach / peak, "peak_kind": peak_kind, "traffic": traffic,
+                     "bytes_per_launch": dom_bytes, "ms_per_launch": dom_ms},
         "kernels": {"expand_ms_per_step": exp_ms, "expand_ms_by_depth": [x / n_k for x in by_depth],
                     "expand_gbs": exp_gbs, "prune_ms": prune_ms,
                     "verify_ms": ver_ms, "verify_gbs": ver_gbs, "step_gbs": step_gbs,
                     "step_frac_of_peak": step_gbs / peak},
         "clocks": clocks,
-        "gpu_launches": args.steps * (D + 3),
+        "gpu_launches": args.steps * (D + 4),  # D expand, 1 prune, 3 verify (prep, stream, residual)
         "e2e": e2e,
         "cpu_baseline": cpu,
     }

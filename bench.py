@@ -267,6 +267,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (a smaller case of the same kernels, for profiling)")
+    ap.add_argument("--depth", type=int, default=0,
+                    help="override the workload's depth (fewer expansion launches of the same shape, for profiling)")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)
 
@@ -276,6 +278,8 @@ def main(argv=None):
     w = synth.WORKLOADS[args.workload]
     if args.batch > 0 and args.batch != w.batch:
         w = dataclasses.replace(w, name=f"{w.name}_b{args.batch}", batch=args.batch)
+    if args.depth > 0 and args.depth != w.depth:
+        w = dataclasses.replace(w, name=f"{w.name}_d{args.depth}", depth=args.depth)
     if args.impl == "reference":
         return run_reference(args, w)
 

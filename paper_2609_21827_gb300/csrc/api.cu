@@ -181,23 +181,22 @@ extern "C" int rheo_expand(const rheo_config* cfg, int32_t d, const void* logits
     const int tpr = tiles_per_row(*cfg);
     const int64_t rows = (int64_t)cfg->batch * a.F;
     const int sms = sm_count();
-    // Launch shape.  Up to one row per SM: every row is cut into P equal
-    // segments (P CTAs, P = SMs / rows), so a CTA holds one segment and P = 1
-    // needs no merge.  More rows: two CTAs per SM, rows cut where the even
-    // split of the tiles falls.
+    // Launch shape: one CTA of 16 warps per SM.  Up to one row per SM: every
+    // row is cut into P equal segments (P CTAs, P = SMs / rows), so a CTA holds
+    // one segment and P = 1 needs no merge.  More rows: one CTA per SM, rows
+    // cut where the even split of the tiles falls.
     int grid;
-    const bool whole = rows <= sms;
-    if (whole) {
+    if (rows <= sms) {
         const int64_t P = std::max<int64_t>(1, std::min<int64_t>(tpr, sms / rows));
         grid = (int)(rows * P);
     } else {
-        grid = (int)std::min<int64_t>(rows * tpr, 2 * (int64_t)sms);
+        grid = (int)std::min<int64_t>(rows * tpr, (int64_t)sms);
     }
     const int segs = max_segments(rows, tpr, grid);
     a.keys_bytes = expand_keys_bytes(segs, cfg->support);
     const size_t smem = expand_smem_bytes(segs, cfg->support);
     if (smem + 8 * 1024 > 227 * 1024) return RHEO_EINVAL;
-    return launch_expand(a, cfg->dtype, rows_aligned(logits, row_stride, *cfg), whole, grid, smem, (cudaStream_t)stream) ==
+    return launch_expand(a, cfg->dtype, rows_aligned(logits, row_stride, *cfg), grid, smem, (cudaStream_t)stream) ==
                    cudaSuccess
                ? RHEO_OK
                : RHEO_ELAUNCH;

@@ -29,8 +29,14 @@ namespace rheo {
 
 namespace {
 
-constexpr int kRegion = 256;   // candidate keys per warp
-constexpr int kVPT = 4;        // 16-byte vectors per thread per tile
+constexpr int kXThreads = 512;  // one CTA of 16 warps per SM
+constexpr int kXWarps = kXThreads / 32;
+constexpr int kRegion = 256;    // candidate keys per warp
+constexpr int kVPT = 4;         // 16-byte vectors per thread per tile
+constexpr int kXTileBytes = kVPT * 16 * kXThreads;  // 32 KiB per tile
+constexpr int kStageCap = 32 * kVPT;  // staged vectors per warp: a whole tile's worth
+// per-warp staging lists while streaming; the bin-ordered list of the top-S sort after
+constexpr int kSpillBytes = kXWarps * kStageCap * (int)(sizeof(uint4) + sizeof(int));
 // two-level histogram of candidate keys: 256 coarse bins (top 8 key bits, two
 // octaves of value each) over 16384 fine bins (top 14 bits, 1/32 octave)
 constexpr int kCoarseBins = 256, kCoarseShift = 56;
@@ -89,21 +95,40 @@ __device__ __noinline__ unsigned long long warp_cut_region(unsigned long long* r
     return thr;
 }
 
-// The tile's vectors of this thread: elements [e0 + (j*kThreads + tid)*VEC, +VEC);
+// Asynchronous 4- and 8-byte copies global -> shared (no register held while
+// they are in flight); cp_async_wait waits for the calling thread's copies.
+__device__ __forceinline__ void cp_async(void* smem, const void* gmem, int bytes) {
+    const unsigned sa = (unsigned)__cvta_generic_to_shared(smem);
+    if (bytes == 8)
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(sa), "l"(gmem) : "memory");
+    else
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(sa), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
+// Per-row values the end of a segment needs (request constants, the parent's
+// gen id and path score), fetched while the row streams.
+struct RowPre {
+    unsigned long long seed, off;
+    float T, ps;
+    int par_g, stage;
+};
+
+// The tile's vectors of this thread: elements [e0 + (j*kXThreads + tid)*VEC, +VEC);
 // positions at or past V read as -inf.
 template <int DT, bool ALIGNED>
 __device__ __forceinline__ void load_tile(uint4 (&v)[kVPT], const char* row, int e0, int V) {
     using E = Elem<DT>;
-    constexpr int TE = kVPT * kThreads * E::VEC;
+    constexpr int TE = kVPT * kXThreads * E::VEC;
     if (ALIGNED && e0 + TE <= V) {  // a whole tile: plain 16-byte loads
 #pragma unroll
         for (int j = 0; j < kVPT; ++j)
-            v[j] = ld_stream(row + ((int64_t)e0 + (j * kThreads + (int)threadIdx.x) * E::VEC) * E::SIZE);
+            v[j] = ld_stream(row + ((int64_t)e0 + (j * kXThreads + (int)threadIdx.x) * E::VEC) * E::SIZE);
         return;
     }
 #pragma unroll
     for (int j = 0; j < kVPT; ++j)
-        v[j] = load_vec<DT, ALIGNED>(row, (int64_t)e0 + (j * kThreads + (int)threadIdx.x) * E::VEC, V);
+        v[j] = load_vec<DT, ALIGNED>(row, (int64_t)e0 + (j * kXThreads + (int)threadIdx.x) * E::VEC, V);
 }
 
 // Append the keys >= thr among get(i), i < n, to sel (at most cap of them);
@@ -112,7 +137,7 @@ template <class Get>
 __device__ __forceinline__ void gather_at_least(Get get, int n, unsigned long long thr, unsigned long long* sel,
                                                 int cap, int* counter) {
     const int lane = threadIdx.x & 31;
-    for (int i0 = 0; i0 < n; i0 += kThreads) {
+    for (int i0 = 0; i0 < n; i0 += kXThreads) {
         const int i = i0 + (int)threadIdx.x;
         const unsigned long long x = i < n ? get(i) : 0ull;
         const bool take = x != 0ull && x >= thr;
@@ -180,18 +205,18 @@ __device__ __forceinline__ void warp_hist_find(const unsigned* coarse, const uns
 // hs.tie_n = 0.  Thread t scans coarse bin 255 - t (a block scan from the top),
 // then one warp scans the 64 fine bins of the coarse bin found.
 __device__ void hist_boundary(const unsigned* coarse, const unsigned* fine, int k, HistSel& hs, Red& red, int& par) {
-    static_assert(kCoarseBins == kThreads, "one coarse bin per thread");
+    static_assert(kCoarseBins <= kXThreads, "one coarse bin per thread");
     const int tid = threadIdx.x, lane = tid & 31;
-    const int cb = kCoarseBins - 1 - tid;
-    const int c = (int)coarse[cb];
+    const int cb = kCoarseBins - 1 - tid;  // negative: no bin
+    const int c = cb >= 0 ? (int)coarse[cb] : 0;
     int total;
-    const int before = red_scan(c, total, red, par);
-    hs.cbefore[cb] = before;
+    const int before = red_scan<kXWarps>(c, total, red, par);
+    if (cb >= 0) hs.cbefore[cb] = before;
     if (tid == 0) {
         hs.bin = -1;
         hs.tie_n = 0;
     }
-    if (total >= k && before < k && before + c >= k) {
+    if (c > 0 && total >= k && before < k && before + c >= k) {
         hs.cbin = cb;
         hs.above = before;
     }
@@ -241,7 +266,7 @@ __device__ int hist_sort_top(Scatter scatter, CoarseCount coarse_count, int k, u
         // bin 255 - t), the 64 fine bins two per lane with a warp scan, from the top
         static_assert(kFinePerCoarse == 64, "two fine bins per lane");
         const int cbl = kCoarseBins - 1 - tid;
-        unsigned todo = __ballot_sync(0xFFFFFFFFu, cbl >= cstar && coarse_count(cbl) > 0);
+        unsigned todo = __ballot_sync(0xFFFFFFFFu, cbl >= 0 && cbl >= cstar && coarse_count(cbl) > 0);
         while (todo) {
             const int L = __ffs(todo) - 1;
             todo &= todo - 1u;
@@ -270,7 +295,7 @@ __device__ int hist_sort_top(Scatter scatter, CoarseCount coarse_count, int k, u
     });
     __syncthreads();
     const int kk = nsel < k ? nsel : k;
-    for (int p = tid; p < nsel; p += kThreads) {
+    for (int p = tid; p < nsel; p += kXThreads) {
         const unsigned long long x = tmp[p];
         const int f = (int)(x >> kFineShift);
         const int start = (f % kFinePerCoarse == kFinePerCoarse - 1) ? hs.cbefore[f / kFinePerCoarse] : (int)fine[f + 1];
@@ -288,7 +313,7 @@ template <class Get>
 __device__ __forceinline__ void block_gather_bin(Get get, int n, int bin, unsigned long long* tmp, int cap,
                                                  HistSel& hs) {
     const int lane = threadIdx.x & 31;
-    for (int i0 = 0; i0 < n; i0 += kThreads) {
+    for (int i0 = 0; i0 < n; i0 += kXThreads) {
         const int i = i0 + (int)threadIdx.x;
         const unsigned long long x = i < n ? get(i) : 0ull;
         const bool take = x != 0ull && (int)(x >> kFineShift) >= bin;
@@ -307,7 +332,7 @@ __device__ int rank_gathered(const unsigned long long* tmp, int k, unsigned long
     __syncthreads();
     const int nsel = hs.tie_n;
     const int kk = nsel < k ? nsel : k;
-    for (int p0 = 0; p0 < nsel; p0 += kThreads / 2) {
+    for (int p0 = 0; p0 < nsel; p0 += kXThreads / 2) {
         const int p = p0 + ((int)threadIdx.x >> 1), h = threadIdx.x & 1;
         const unsigned long long x = p < nsel ? tmp[p] : 0ull;
         int rank = 0;
@@ -328,17 +353,15 @@ __device__ int rank_gathered(const unsigned long long* tmp, int k, unsigned long
     return kk;
 }
 
-// Slow insertion path of one tile's candidates (pend: this lane's element
-// bits; the lanes' vectors are in wspill): one candidate per lane and round,
-// keys below theta dropped, the region cut to its S best whenever it fills.
+// Slow insertion path (pend: this lane's element bits of its vector vv, whose
+// first element is eidx): one candidate per lane and round, keys below theta
+// dropped, the region cut to its S best whenever it fills.
 template <int DT>
-__device__ __noinline__ void insert_rounds(unsigned long long* region, int& cnt, uint32_t pend, const uint4* wspill,
-                                           int e0, unsigned long long& theta, int S, unsigned* fine,
-                                           unsigned* coarse, unsigned long long* s_theta) {
+__device__ __forceinline__ void insert_rounds(unsigned long long* region, int& cnt, uint32_t pend, uint4 vv, int eidx,
+                                           unsigned long long& theta, int S, unsigned* fine, unsigned* coarse,
+                                           unsigned long long* s_theta) {
     using E = Elem<DT>;
-    constexpr int VEC = E::VEC;
-    const int lane = threadIdx.x & 31, tid = threadIdx.x;
-    const uint32_t* wv0 = reinterpret_cast<const uint32_t*>(wspill);
+    const int lane = threadIdx.x & 31;
     while (__any_sync(0xFFFFFFFFu, pend != 0u)) {
         if (cnt > kRegion - 32) {
             const unsigned long long thr = warp_cut_region(region, cnt, S, fine, coarse);
@@ -347,12 +370,9 @@ __device__ __noinline__ void insert_rounds(unsigned long long* region, int& cnt,
         }
         unsigned long long x = 0ull;
         if (pend) {
-            const int q = __ffs(pend) - 1;
+            const int i = __ffs(pend) - 1;
             pend &= pend - 1u;
-            const int j = q / VEC, i = q % VEC;
-            const uint32_t* wv = wv0 + (j * 32 + lane) * 4;
-            const uint32_t raw = (DT == 0) ? wv[i] : ((wv[i >> 1] >> ((i & 1) * 16)) & 0xFFFFu);
-            x = make_key(E::key(raw), (int64_t)e0 + (j * kThreads + tid) * VEC + i);
+            x = make_key(E::key(E::raw(vv, i)), (int64_t)eidx + i);
             if (x < theta) x = 0ull;
         }
         const unsigned bal = __ballot_sync(0xFFFFFFFFu, x != 0ull);
@@ -365,16 +385,68 @@ __device__ __noinline__ void insert_rounds(unsigned long long* region, int& cnt,
     }
 }
 
+// One warp inserts its staged vectors (sv[0, n), first elements si[]) into its
+// candidate region: every element at or above theta (as it stands now) of
+// the row's first V elements becomes a key, counted in both histograms; one
+// vector per lane and round.
+template <int DT>
+__device__ __forceinline__ void stage_flush(unsigned long long* region, int& cnt, const uint4* sv, const int* si, int n,
+                                         int V, unsigned long long& theta, int S, unsigned* fine, unsigned* coarse,
+                                         unsigned long long* s_theta) {
+    using E = Elem<DT>;
+    using W = Vec<DT>;
+    constexpr int VEC = E::VEC;
+    const int lane = threadIdx.x & 31;
+    for (int k0 = 0; k0 < n; k0 += 32) {
+        const float thv = E::threshold_value((uint32_t)(theta >> 32));
+        const uint32_t t2 = (DT == 0) ? __float_as_uint(thv)
+                                      : ((__float_as_uint(thv) >> 16) | (__float_as_uint(thv) & 0xFFFF0000u));
+        const int k = k0 + lane;
+        uint4 vv = make_uint4(0u, 0u, 0u, 0u);
+        int eidx = 0;
+        uint32_t pend = 0u;
+        if (k < n) {
+            vv = sv[k];
+            eidx = si[k];
+            pend = W::ge_bits(vv, t2);
+            const int left = V - eidx;  // elements of this vector inside the row
+            if (left < VEC) pend &= (left > 0) ? ((1u << left) - 1u) : 0u;
+        }
+        const int c = __popc(pend);
+        int incl = c;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        const int total = __shfl_sync(0xFFFFFFFFu, incl, 31);
+        if (cnt + total <= kRegion) {
+            int pos = cnt + incl - c;
+            for (uint32_t mm = pend; mm; mm &= mm - 1u) {
+                const int i = __ffs(mm) - 1;
+                const unsigned long long x = make_key(E::key(E::raw(vv, i)), (int64_t)eidx + i);
+                region[pos++] = x;
+                atomicAdd(&fine[(unsigned)(x >> kFineShift)], 1u);
+                atomicAdd(&coarse[(unsigned)(x >> kCoarseShift)], 1u);
+            }
+            cnt += total;
+        } else {
+            insert_rounds<DT>(region, cnt, pend, vv, eidx, theta, S, fine, coarse, s_theta);
+        }
+    }
+    __syncwarp();
+}
+
 }  // namespace
 
-template <int DT, bool ALIGNED, int NS>
-__global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const ExpandArgs a) {
+template <int DT, bool ALIGNED>
+__global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a) {
     grid_dependency_begin();
     using E = Elem<DT>;
     using W = Vec<DT>;
     constexpr int VEC = E::VEC;
-    constexpr int TE = kTileBytes / E::SIZE;  // elements per tile
-    static_assert(TE == kVPT * VEC * kThreads, "tile layout");
+    constexpr int TE = kXTileBytes / E::SIZE;  // elements per tile
+    static_assert(TE == kVPT * VEC * kXThreads, "tile layout");
     constexpr float kLog2e = 1.4426950408889634f;
     extern __shared__ __align__(128) unsigned char dsm[];
     // per-warp candidate regions; after a segment's selection the same space
@@ -382,46 +454,80 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
     unsigned long long* keys = reinterpret_cast<unsigned long long*>(dsm);
     // per-warp copy of the lanes' vectors of a tile that has candidates
     uint4* spill = reinterpret_cast<uint4*>(dsm + a.keys_bytes);
-    unsigned* fine = reinterpret_cast<unsigned*>(dsm + a.keys_bytes + sizeof(uint4) * kWarps * 32 * kVPT);
+    unsigned* fine = reinterpret_cast<unsigned*>(dsm + a.keys_bytes + kSpillBytes);
     unsigned* coarse = fine + kFineBins;
     // the spill area doubles as the bin-ordered list of the top-S sort
     unsigned long long* tmpk = reinterpret_cast<unsigned long long*>(spill);
-    constexpr int kTmpCap = kWarps * 32 * kVPT * (int)sizeof(uint4) / (int)sizeof(unsigned long long);
+    constexpr int kTmpCap = kSpillBytes / (int)sizeof(unsigned long long);
     __shared__ unsigned long long s_theta;
-    __shared__ uint32_t s_wb[kWarps];
-    __shared__ int s_rcount[kWarps];
+    __shared__ uint32_t s_wb[kXWarps];
+    __shared__ int s_rcount[kXWarps];
     __shared__ BlockScratch bs;
     __shared__ Red red;
     __shared__ E2Smem e2;
     __shared__ HistSel hs;
     __shared__ unsigned s_hist[kRadixBins];
     __shared__ SelScratch s_sel;
+    __shared__ RowPre s_pre;
 
     const Dims& n = a.n;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int V = n.V, S = n.S, K = n.K, m = n.m, TL = n.TL;
     const int tpr = (V + TE - 1) / TE;
-    const int kb = (S + kWarps - 1) / kWarps;  // per-warp share of S in the bounds
+    const int kb = (S + kXWarps - 1) / kXWarps;  // per-warp share of S in the bounds
     const TileSplit sp{(int64_t)n.B * a.F * tpr, (int)gridDim.x};
     const int64_t t0 = sp.begin(blockIdx.x), t1 = sp.begin(blockIdx.x + 1);
     unsigned long long* region = keys + warp * kRegion;
-    uint4* wspill = spill + warp * (32 * kVPT);
+    // per-warp staging list of vectors holding candidates (in the spill area)
+    static_assert(kXWarps * kStageCap * (sizeof(uint4) + sizeof(int)) <= kSpillBytes, "staging fits the spill area");
+    uint4* stage_v = spill + warp * kStageCap;
+    int* stage_i = reinterpret_cast<int*>(spill + kXWarps * kStageCap) + warp * kStageCap;
+    int scnt = 0;  // staged vectors of this warp (warp-uniform)
     int par = 0;
 
     if (tid == 0) s_theta = 0ull;
 
     // per-segment state; cnt, theta and seg_valid are warp-uniform
-    float mu = -INFINITY, sum = 0.0f;
+    float mu = -INFINITY;
+    unsigned long long sum2 = 0ull;  // the running sum as a pair of fp32 partial sums
     unsigned long long theta = 0ull;
     int cnt = 0, seg_tiles = 0;
     int64_t seg_valid = 0;
 
+    // tid 0 starts the copies of the row's constants and, on the second tile, of
+    // its parent's score (which needs the parent's gen id from the frontier)
+    auto prefetch_row = [&](int64_t r) {
+        if (tid != 0) return;
+        const int b = (int)(r / a.F), f = (int)(r % a.F);
+        cp_async(&s_pre.T, a.T + b, 4);
+        cp_async(&s_pre.seed, a.seed + b, 8);
+        cp_async(&s_pre.off, a.offset + b, 8);
+        if (a.d > 1) {
+            cp_async(&s_pre.par_g, a.tree.frontier + (int64_t)b * K + f, 4);
+            s_pre.stage = 1;
+        } else {  // the root: nothing to fetch
+            s_pre.par_g = 0;
+            s_pre.ps = 0.0f;
+            s_pre.stage = 0;
+        }
+    };
+    auto prefetch_parent = [&](int64_t r) {  // tid 0, after the frontier entry arrived
+        cp_async_wait();
+        if (s_pre.stage != 1) return;
+        const int b = (int)(r / a.F);
+        const int pg = s_pre.par_g;
+        s_pre.stage = 2;
+        if (pg >= 0 && pg < n.G1)
+            cp_async(&s_pre.ps, a.tree.score + (int64_t)b * n.G1 + pg, 4);
+        else
+            s_pre.ps = 0.0f;  // reported as an internal error at the segment's end
+    };
     auto seg_begin = [&]() {
         mu = -INFINITY;
-        sum = 0.0f;
+        sum2 = 0ull;
         seg_valid = 0;
         cnt = 0;
-        for (int i = tid; i < (kFineBins + kCoarseBins) / 4; i += kThreads)
+        for (int i = tid; i < (kFineBins + kCoarseBins) / 4; i += kXThreads)
             reinterpret_cast<uint4*>(fine)[i] = make_uint4(0u, 0u, 0u, 0u);
     };
     // running partition sum at T = 1 (online max); mu is also the running
@@ -429,15 +535,23 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
     auto tile_sum = [&](const uint4 (&v)[kVPT], float (&vm)[kVPT]) {
 #pragma unroll
         for (int j = 0; j < kVPT; ++j) vm[j] = W::vmax(v[j]);
-        const float tmax = fmaxf(fmaxf(vm[0], vm[1]), fmaxf(vm[2], vm[3]));
+        float tmax = vm[0];
+#pragma unroll
+        for (int j = 1; j < kVPT; ++j) tmax = fmaxf(tmax, vm[j]);
         if (tmax > mu) {
-            if (mu != -INFINITY) sum *= fast_exp2((mu - tmax) * kLog2e);
+            if (mu != -INFINITY) {
+                const float rs = fast_exp2((mu - tmax) * kLog2e);
+                sum2 = f2_mul(sum2, f2_pack(rs, rs));
+            }
             mu = tmax;
         }
         if (mu != -INFINITY) {
             const float mc = mu * kLog2e;
-            sum += (W::vexp(v[0], kLog2e, mc) + W::vexp(v[1], kLog2e, mc)) +
-                   (W::vexp(v[2], kLog2e, mc) + W::vexp(v[3], kLog2e, mc));
+            const unsigned long long c2 = f2_pack(kLog2e, kLog2e), n2 = f2_pack(-mc, -mc);
+            unsigned long long t = W::vexp2(v[0], c2, n2);
+#pragma unroll
+            for (int j = 1; j < kVPT; ++j) t = f2_add(t, W::vexp2(v[j], c2, n2));
+            sum2 = f2_add(sum2, t);
         }
     };
     // The bound theta.  On the first step of a segment: every warp's kb-th
@@ -463,9 +577,9 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
             __syncthreads();
             uint32_t b = s_wb[0];
 #pragma unroll
-            for (int w = 1; w < kWarps; ++w) b = min(b, s_wb[w]);
+            for (int w = 1; w < kXWarps; ++w) b = min(b, s_wb[w]);
             theta = (unsigned long long)b << 32;
-        } else if (seg_tiles % kWarps == warp) {
+        } else if (seg_tiles % kXWarps == warp) {
             int bin, above;
             warp_hist_find(coarse, fine, S, bin, above);
             if (bin >= 0) {
@@ -480,57 +594,45 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
     // candidates of one tile: elements whose value reaches theta's (a superset
     // of the keys >= theta; the final selection is exact).  Every lane writes its
     // own at offsets from a warp scan.
-    auto tile_candidates = [&](const uint4 (&v)[kVPT], const float (&vm)[kVPT], int e0, int ne) {
+    auto tile_candidates = [&](const uint4 (&v)[kVPT], const float (&vm)[kVPT], int e0) {
         const float thv = E::threshold_value((uint32_t)(theta >> 32));
-        // the bound in the element's own format (bf16: a pair), compared packed
-        const uint32_t t2 = (DT == 0) ? __float_as_uint(thv)
-                                      : ((__float_as_uint(thv) >> 16) | (__float_as_uint(thv) & 0xFFFF0000u));
-        uint32_t pend = 0u;
+        // a vector whose maximum reaches theta is staged as it is (its elements
+        // are screened when the list is flushed): a vote per vector row of the
+        // tile, one store per staged vector
+        unsigned bal[kVPT];
+        int total = 0;
 #pragma unroll
         for (int j = 0; j < kVPT; ++j) {
-            uint32_t bits = W::ge_bits(v[j], t2);
-            const int left = ne - (j * kThreads + tid) * VEC;  // elements of this vector inside the tile
-            if (left < VEC) bits &= (left > 0) ? ((1u << left) - 1u) : 0u;
-            pend |= bits << (j * VEC);
+            bal[j] = __ballot_sync(0xFFFFFFFFu, vm[j] >= thv);
+            total += __popc(bal[j]);
         }
-        if (!__any_sync(0xFFFFFFFFu, pend != 0u)) return;
-#pragma unroll
-        for (int j = 0; j < kVPT; ++j) wspill[j * 32 + lane] = v[j];
-        const int c = __popc(pend);
-        int incl = c;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-            if (lane >= o) incl += y;
+        if (total == 0) return;
+        if (scnt + total > kStageCap) {
+            stage_flush<DT>(region, cnt, stage_v, stage_i, scnt, V, theta, S, fine, coarse, &s_theta);
+            scnt = 0;
         }
-        const int total = __shfl_sync(0xFFFFFFFFu, incl, 31);
-        if (cnt + total <= kRegion) {
-            const uint32_t* wv0 = reinterpret_cast<const uint32_t*>(wspill);
-            int pos = cnt + incl - c;
-            for (uint32_t mm = pend; mm; mm &= mm - 1u) {
-                const int q = __ffs(mm) - 1;
-                const int j = q / VEC, i = q % VEC;
-                const uint32_t* wv = wv0 + (j * 32 + lane) * 4;
-                const uint32_t raw = (DT == 0) ? wv[i] : ((wv[i >> 1] >> ((i & 1) * 16)) & 0xFFFFu);
-                const unsigned long long x = make_key(E::key(raw), (int64_t)e0 + (j * kThreads + tid) * VEC + i);
-                region[pos++] = x;
-                atomicAdd(&fine[(unsigned)(x >> kFineShift)], 1u);
-                atomicAdd(&coarse[(unsigned)(x >> kCoarseShift)], 1u);
+#pragma unroll
+        for (int j = 0; j < kVPT; ++j) {
+            if ((bal[j] >> lane) & 1u) {
+                const int p = scnt + __popc(bal[j] & ((1u << lane) - 1u));
+                stage_v[p] = v[j];
+                stage_i[p] = e0 + (j * kXThreads + tid) * VEC;
             }
-            cnt += total;
-        } else {
-            // the region would overflow: one candidate per lane and round, keys
-            // below theta dropped, the region cut whenever it fills
-            insert_rounds<DT>(region, cnt, pend, wspill, e0, theta, S, fine, coarse, &s_theta);
+            scnt += __popc(bal[j]);
         }
-        __syncwarp();
     };
     // end of the segment of row r that this CTA holds
     auto segment_end = [&](int64_t r) {
         // ---- end of segment: exact top-S keys ------------------------------------
+        if (tid == 0) {  // the row's constants have landed (or land now)
+            prefetch_parent(r);
+            cp_async_wait();
+        }
+        if (scnt > 0) stage_flush<DT>(region, cnt, stage_v, stage_i, scnt, V, theta, S, fine, coarse, &s_theta);
+        scnt = 0;
         if (lane == 0) s_rcount[warp] = cnt;
         float Ms;
-        const FF Ss = red_partition(mu, sum, kLog2e, Ms, red, par);  // its barrier also publishes the counts
+        const FF Ss = red_partition<kXWarps>(mu, f2_fold(sum2), kLog2e, Ms, red, par);  // its barrier also publishes the counts
         if (tid == 0) s_theta = 0ull;  // every warp is past its last cut: ready for the next segment
         const int target = (int)min((int64_t)S, seg_valid);
         auto rkey = [&](int i) -> unsigned long long {
@@ -546,10 +648,10 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
                 },
                 [&](int c) { return coarse[c]; }, target, fine, tmpk, e2.sorted, hs);
         } else {  // a tie class too large for the list
-            const unsigned long long thr = block_kth_key(rkey, kWarps * kRegion, target, s_hist, s_sel);
+            const unsigned long long thr = block_kth_key<kXThreads>(rkey, kXWarps * kRegion, target, s_hist, s_sel);
             if (tid == 0) hs.tie_n = 0;
             __syncthreads();
-            gather_at_least(rkey, kWarps * kRegion, thr, tmpk, target, &hs.tie_n);
+            gather_at_least(rkey, kXWarps * kRegion, thr, tmpk, target, &hs.tie_n);
             written = rank_gathered(tmpk, target, e2.sorted, hs);
         }
         const int first_owner = sp.owner(r * tpr);
@@ -569,7 +671,7 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
             }
         } else {
             unsigned long long* out = a.seg_keys + ((int64_t)r * tpr + seg) * S;
-            for (int i = tid; i < S; i += kThreads) out[i] = i < written ? e2.sorted[i] : 0ull;
+            for (int i = tid; i < S; i += kXThreads) out[i] = i < written ? e2.sorted[i] : 0ull;
             if (tid == 0) {
                 a.seg_mu[(int64_t)r * tpr + seg] = Ms;
                 a.seg_sum[2 * ((int64_t)r * tpr + seg)] = Ss.hi;
@@ -580,10 +682,10 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
             // ---- last segment of row r: merge the segments' lists and sums ---------
             const int nkeys = nseg * S;
             const unsigned long long* rk = a.seg_keys + (int64_t)r * tpr * S;
-            for (int i = tid; i < (kFineBins + kCoarseBins) / 4; i += kThreads)
+            for (int i = tid; i < (kFineBins + kCoarseBins) / 4; i += kXThreads)
                 reinterpret_cast<uint4*>(fine)[i] = make_uint4(0u, 0u, 0u, 0u);
             __syncthreads();
-            for (int i = tid; i < nkeys; i += kThreads) {
+            for (int i = tid; i < nkeys; i += kXThreads) {
                 const unsigned long long x = __ldcg(rk + i);
                 keys[i] = x;
                 if (x) {
@@ -598,12 +700,12 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
             if (hs.bin < 0 || hs.above + (int)fine[hs.bin] <= kTmpCap) {
                 got = hist_sort_top(
                     [&](auto put) {
-                        for (int i = tid; i < nkeys; i += kThreads)
+                        for (int i = tid; i < nkeys; i += kXThreads)
                             if (keys[i]) put(keys[i]);
                     },
                     [&](int c) { return coarse[c]; }, S, fine, tmpk, e2.sorted, hs);
             } else {
-                const unsigned long long thr = block_kth_key(mkey, nkeys, S, s_hist, s_sel);
+                const unsigned long long thr = block_kth_key<kXThreads>(mkey, nkeys, S, s_hist, s_sel);
                 if (tid == 0) hs.tie_n = 0;
                 __syncthreads();
                 gather_at_least(mkey, nkeys, thr, tmpk, S, &hs.tie_n);
@@ -643,10 +745,10 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
         }
         __syncthreads();
 
-        const float T = a.T[b];
-        const uint64_t seed = a.seed[b], off = a.offset[b];
+        const float T = s_pre.T;
+        const uint64_t seed = s_pre.seed, off = s_pre.off;
         const int64_t nb = (int64_t)b * n.G1;
-        int64_t par_g = (a.d == 1) ? 0 : (int64_t)a.tree.frontier[(int64_t)b * K + f];
+        int64_t par_g = s_pre.par_g;
         if (par_g < 0 || par_g >= n.G1) {  // frontier never written for this tree
             if (tid == 0) atomicOr(a.status, kStInternal);
             par_g = 0;
@@ -657,7 +759,7 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
         // tempered tail q~ = softmax(l / T) over support ranks m+1..S; Y by Gumbel-max
         const float tau = (tid < TL) ? __fdiv_rn(e2.l[m + tid], T) : -INFINITY;
         const float mt = __fdiv_rn(e2.l[m], T);  // the support is sorted: rank m is the tail's maximum
-        const FF st = red_sum_ff(FF{(tid < TL && mt > -INFINITY) ? expf(tau - mt) : 0.0f, 0.0f}, red, par);
+        const FF st = red_sum_ff<kXWarps>(FF{(tid < TL && mt > -INFINITY) ? expf(tau - mt) : 0.0f, 0.0f}, red, par);
         const FF lse_tail = ff_add(ff_log(st), mt);
         unsigned long long pack = 0ull;
         if (tid < TL) {
@@ -666,7 +768,7 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
             const float key = __fadd_rn(tau, g);
             if (key > -INFINITY) pack = make_key(ord_f32(key), tid);
         }
-        const unsigned long long bestp = red_max_u64(pack, red, par);
+        const unsigned long long bestp = red_max_u64<kXWarps>(pack, red, par);
         if (tid == 0) {
             e2.best = bestp ? (int)(0xFFFFFFFFu - (uint32_t)bestp) : 0;
             if (e2.bad) atomicOr(a.status, kStInternal);
@@ -714,7 +816,7 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
                 const int qf = j - m - 1;
                 rank = m + qf + (qf >= best ? 1 : 0); lpj = e2.lq0[rank]; st8 = kSlotFill;
             }
-            const float ps = (a.d == 1) ? 0.0f : a.tree.score[nb + par_g];
+            const float ps = s_pre.ps;
             const int64_t g = nb + g0 + j;
             a.tree.token[g] = e2.id[rank];
             a.tree.parent[g] = (int32_t)par_g;
@@ -736,7 +838,7 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
         {
             const int nn = a.F * (K + 1);
             const int64_t base = depth_base(K, a.d);
-            if (nn <= kThreads) {
+            if (nn <= kXThreads) {
                 // rank of every candidate; the K best, written in gen-id order
                 const unsigned long long x =
                     tid < nn ? make_key(ord_f32(__ldcg(a.tree.score + nb + base + tid)), base + tid) : 0ull;
@@ -747,20 +849,20 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
                     for (int j = 0; j < nn; ++j) rank += keys[j] > x;
                 const bool take = tid < nn && rank < K;
                 int total;
-                const int pos = red_scan(take ? 1 : 0, total, red, par);
+                const int pos = red_scan<kXWarps>(take ? 1 : 0, total, red, par);
                 if (take && pos < K) a.tree.frontier[(int64_t)b * K + pos] = (int32_t)(base + tid);
                 if (tid == 0 && total != K) atomicOr(a.status, kStInternal);
             } else {
                 auto key_at = [&](int i) -> unsigned long long {
                     return make_key(ord_f32(__ldcg(a.tree.score + nb + base + i)), base + i);
                 };
-                const unsigned long long fthr = block_kth_key(key_at, nn, K, s_hist, s_sel);
-                const int per = (nn + kThreads - 1) / kThreads;
+                const unsigned long long fthr = block_kth_key<kXThreads>(key_at, nn, K, s_hist, s_sel);
+                const int per = (nn + kXThreads - 1) / kXThreads;
                 const int lo = min(nn, tid * per), hi = min(nn, lo + per);
                 int c = 0;
                 for (int i = lo; i < hi; ++i) c += key_at(i) >= fthr;
                 int total;
-                int pos = red_scan(c, total, red, par);
+                int pos = red_scan<kXWarps>(c, total, red, par);
                 for (int i = lo; i < hi; ++i)
                     if (key_at(i) >= fthr) {
                         if (pos < K) a.tree.frontier[(int64_t)b * K + pos] = (int32_t)(base + i);
@@ -772,7 +874,7 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
         }
     };
 
-    if (NS == 1) {
+    {
         // the CTA's tiles in order; segments end at row boundaries
         int64_t r = t0 / tpr;
         int tt = (int)(t0 % tpr);
@@ -794,76 +896,43 @@ __global__ void __launch_bounds__(kThreads, NS == 1 ? 2 : 1) expand_kernel(const
                 const bool wrap = (tt + 1 == tpr);
                 load_tile<DT, ALIGNED>(nxt, a.logits + (r + (wrap ? 1 : 0)) * a.row_stride_bytes, wrap ? 0 : e0 + TE, V);
             }
-            if (seg_first) seg_begin();
+            if (seg_first) {
+                prefetch_row(r);
+                seg_begin();
+            } else if (tid == 0 && s_pre.stage == 1) {
+                prefetch_parent(r);
+            }
             float vm[kVPT];
             tile_sum(v, vm);
             refresh(seg_first);
             seg_valid += ne;
-            tile_candidates(v, vm, e0, ne);
+            tile_candidates(v, vm, e0);
             if (seg_last) segment_end(r);
         }
-    } else {
-        // the CTA's tiles lie in one row: its two halves are streamed side by
-        // side, two tiles in flight per step
-        if (t0 >= t1) return;
-        const int64_t r = t0 / tpr;
-        const char* row = a.logits + r * a.row_stride_bytes;
-        const int ta = (int)(t0 % tpr);
-        const int len = (int)(t1 - t0), la = (len + 1) / 2, tb = ta + la, lb = len - la;
-        uint4 nxa[kVPT], nxb[kVPT];
-        load_tile<DT, ALIGNED>(nxa, row, ta * TE, V);
-        if (lb > 0) load_tile<DT, ALIGNED>(nxb, row, tb * TE, V);
-        seg_begin();
-        for (int i = 0; i < la; ++i) {
-            const bool hb = i < lb;
-            const int ea = (ta + i) * TE, eb = (tb + i) * TE;
-            const int na = min(TE, V - ea), nb = hb ? min(TE, V - eb) : 0;
-            uint4 va[kVPT], vb[kVPT];
-#pragma unroll
-            for (int j = 0; j < kVPT; ++j) {
-                va[j] = nxa[j];
-                vb[j] = nxb[j];
-            }
-            if (i + 1 < la) load_tile<DT, ALIGNED>(nxa, row, ea + TE, V);
-            if (i + 1 < lb) load_tile<DT, ALIGNED>(nxb, row, eb + TE, V);
-            float vma[kVPT], vmb[kVPT];
-            tile_sum(va, vma);
-            if (hb) tile_sum(vb, vmb);
-            refresh(i == 0);
-            seg_valid += na + nb;
-            tile_candidates(va, vma, ea, na);
-            if (hb) tile_candidates(vb, vmb, eb, nb);
-        }
-        segment_end(r);
     }
 }
 
-cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, bool whole, int grid, size_t smem,
-                          cudaStream_t s) {
+cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, int grid, size_t smem, cudaStream_t s) {
     auto go = [&](auto kern) {
         cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (err != cudaSuccess) return err;
-        return launch_dependent(kern, dim3(grid), dim3(kThreads), smem, s, a);
+        return launch_dependent(kern, dim3(grid), dim3(kXThreads), smem, s, a);
     };
-    if (whole) {
-        if (dtype == 1) return aligned ? go(expand_kernel<1, true, 2>) : go(expand_kernel<1, false, 2>);
-        return aligned ? go(expand_kernel<0, true, 2>) : go(expand_kernel<0, false, 2>);
-    }
-    if (dtype == 1) return aligned ? go(expand_kernel<1, true, 1>) : go(expand_kernel<1, false, 1>);
-    return aligned ? go(expand_kernel<0, true, 1>) : go(expand_kernel<0, false, 1>);
+    if (dtype == 1) return aligned ? go(expand_kernel<1, true>) : go(expand_kernel<1, false>);
+    return aligned ? go(expand_kernel<0, true>) : go(expand_kernel<0, false>);
 }
 
 size_t expand_keys_bytes(int max_segments, int support) {
-    size_t keys = (size_t)kWarps * kRegion;
+    size_t keys = (size_t)kXWarps * kRegion;
     if ((size_t)max_segments * support > keys) keys = (size_t)max_segments * support;
     return (sizeof(unsigned long long) * keys + 127) & ~(size_t)127;  // the spill area after it is 16-byte aligned
 }
 
 size_t expand_smem_bytes(int max_segments, int support) {
-    return expand_keys_bytes(max_segments, support) + sizeof(uint4) * kWarps * 32 * kVPT +
+    return expand_keys_bytes(max_segments, support) + kSpillBytes +
            sizeof(unsigned) * (kFineBins + kCoarseBins);
 }
 
-int expand_tile_elems(int dtype) { return kTileBytes / (dtype == 1 ? 2 : 4); }
+int expand_tile_elems(int dtype) { return kXTileBytes / (dtype == 1 ? 2 : 4); }
 
 }  // namespace rheo

@@ -14,6 +14,7 @@ namespace rheo {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
+constexpr int kMaxWarps = 16;  // largest block of the path (512 threads); scratch is sized for it
 constexpr int kNV = 8;                                 // 128-bit loads per thread per chunk
 constexpr int kChunkBytes = kThreads * kNV * 16;       // 32 KiB per CTA
 constexpr int kMaxSupport = 128;
@@ -138,6 +139,41 @@ __device__ __forceinline__ float fast_exp2(float x) {
     return y;
 }
 
+// Pairs of fp32 values in one 64-bit register, operated on two at a time by the
+// packed fp32 instructions of sm_100+ (same per-element rounding as the scalar
+// fma / add / mul).
+__device__ __forceinline__ unsigned long long f2_pack(float a, float b) {
+    unsigned long long r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+    return r;
+}
+__device__ __forceinline__ float f2_fold(unsigned long long x) {  // a + b
+    float a, b;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(x));
+    return a + b;
+}
+__device__ __forceinline__ unsigned long long f2_fma(unsigned long long a, unsigned long long b, unsigned long long c) {
+    unsigned long long r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+__device__ __forceinline__ unsigned long long f2_add(unsigned long long a, unsigned long long b) {
+    unsigned long long r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ unsigned long long f2_mul(unsigned long long a, unsigned long long b) {
+    unsigned long long r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+// (2^a, 2^b) of a pair
+__device__ __forceinline__ unsigned long long f2_exp2(unsigned long long x) {
+    float a, b;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(x));
+    return f2_pack(fast_exp2(a), fast_exp2(b));
+}
+
 // ---------------------------------------------------------------------------
 // 16-byte vectors of logits: max, partition-sum terms, tail masking
 // ---------------------------------------------------------------------------
@@ -162,6 +198,15 @@ template <> struct Vec<1> {
         const float a2 = fast_exp2(fmaf(bf_lo(v.z), c, -mc)) + fast_exp2(fmaf(bf_hi(v.z), c, -mc));
         const float a3 = fast_exp2(fmaf(bf_lo(v.w), c, -mc)) + fast_exp2(fmaf(bf_hi(v.w), c, -mc));
         return (a0 + a1) + (a2 + a3);
+    }
+    // the same sum as a pair (x c - mc by packed fma; c2 = (c, c), nmc2 = (-mc, -mc))
+    __device__ static __forceinline__ unsigned long long vexp2(const uint4& v, unsigned long long c2,
+                                                              unsigned long long nmc2) {
+        const unsigned long long e0 = f2_exp2(f2_fma(f2_pack(bf_lo(v.x), bf_hi(v.x)), c2, nmc2));
+        const unsigned long long e1 = f2_exp2(f2_fma(f2_pack(bf_lo(v.y), bf_hi(v.y)), c2, nmc2));
+        const unsigned long long e2 = f2_exp2(f2_fma(f2_pack(bf_lo(v.z), bf_hi(v.z)), c2, nmc2));
+        const unsigned long long e3 = f2_exp2(f2_fma(f2_pack(bf_lo(v.w), bf_hi(v.w)), c2, nmc2));
+        return f2_add(f2_add(e0, e1), f2_add(e2, e3));
     }
     // bit i set when element i is >= t (t2: t as a bf16 pair; false for NaN)
     __device__ static __forceinline__ uint32_t ge_bits(const uint4& v, uint32_t t2) {
@@ -189,6 +234,14 @@ template <> struct Vec<0> {
         const float a0 = fast_exp2(fmaf(__uint_as_float(v.x), c, -mc)) + fast_exp2(fmaf(__uint_as_float(v.y), c, -mc));
         const float a1 = fast_exp2(fmaf(__uint_as_float(v.z), c, -mc)) + fast_exp2(fmaf(__uint_as_float(v.w), c, -mc));
         return a0 + a1;
+    }
+    __device__ static __forceinline__ unsigned long long vexp2(const uint4& v, unsigned long long c2,
+                                                              unsigned long long nmc2) {
+        const unsigned long long e0 =
+            f2_exp2(f2_fma(f2_pack(__uint_as_float(v.x), __uint_as_float(v.y)), c2, nmc2));
+        const unsigned long long e1 =
+            f2_exp2(f2_fma(f2_pack(__uint_as_float(v.z), __uint_as_float(v.w)), c2, nmc2));
+        return f2_add(e0, e1);
     }
     __device__ static __forceinline__ uint32_t ge_bits(const uint4& v, uint32_t t2) {
         const float t = __uint_as_float(t2);
@@ -241,16 +294,17 @@ __device__ __forceinline__ float uniform(uint64_t seed, uint64_t offset, int tag
 __device__ __forceinline__ float gumbel(float u) { return -logf(-logf(u)); }
 
 // ---------------------------------------------------------------------------
-// block reductions (kThreads threads, all must call)
+// block reductions (NW warps, all threads must call; NW = kWarps by default)
 // ---------------------------------------------------------------------------
 struct BlockScratch {
-    int ired[2][kWarps];
-    float fred[kWarps];
-    float fred2[kWarps];
-    unsigned long long ured[kWarps];
+    int ired[2][kMaxWarps];
+    float fred[kMaxWarps];
+    float fred2[kMaxWarps];
+    unsigned long long ured[kMaxWarps];
     int flag;
 };
 
+template <int NW = kWarps>
 __device__ __forceinline__ int block_sum_int(int v, BlockScratch& s, int& parity) {
     v = __reduce_add_sync(0xFFFFFFFFu, v);
     int* buf = s.ired[parity];
@@ -259,7 +313,7 @@ __device__ __forceinline__ int block_sum_int(int v, BlockScratch& s, int& parity
     __syncthreads();
     int t = 0;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) t += buf[w];
+    for (int w = 0; w < NW; ++w) t += buf[w];
     return t;
 }
 
@@ -272,6 +326,7 @@ __device__ __forceinline__ unsigned long long warp_max_u64(unsigned long long v)
     return v;
 }
 
+template <int NW = kWarps>
 __device__ __forceinline__ unsigned long long block_max_u64(unsigned long long v, BlockScratch& s) {
     v = warp_max_u64(v);
     __syncthreads();
@@ -279,10 +334,11 @@ __device__ __forceinline__ unsigned long long block_max_u64(unsigned long long v
     __syncthreads();
     unsigned long long t = 0;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) t = s.ured[w] > t ? s.ured[w] : t;
+    for (int w = 0; w < NW; ++w) t = s.ured[w] > t ? s.ured[w] : t;
     return t;
 }
 
+template <int NW = kWarps>
 __device__ __forceinline__ unsigned long long block_and_or_u64(unsigned long long v, bool want_or,
                                                                BlockScratch& s) {
     unsigned lo = (unsigned)v, hi = (unsigned)(v >> 32);
@@ -299,11 +355,12 @@ __device__ __forceinline__ unsigned long long block_and_or_u64(unsigned long lon
     __syncthreads();
     unsigned long long t = want_or ? 0ull : ~0ull;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) t = want_or ? (t | s.ured[w]) : (t & s.ured[w]);
+    for (int w = 0; w < NW; ++w) t = want_or ? (t | s.ured[w]) : (t & s.ured[w]);
     return t;
 }
 
 // block-wide maximum (all threads get it)
+template <int NW = kWarps>
 __device__ __forceinline__ float block_max_f32(float v, BlockScratch& s) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
@@ -312,7 +369,7 @@ __device__ __forceinline__ float block_max_f32(float v, BlockScratch& s) {
     __syncthreads();
     float m = s.fred[0];
 #pragma unroll
-    for (int w = 1; w < kWarps; ++w) m = fmaxf(m, s.fred[w]);
+    for (int w = 1; w < NW; ++w) m = fmaxf(m, s.fred[w]);
     return m;
 }
 
@@ -370,6 +427,7 @@ __device__ __forceinline__ bool ff_le(FF x, float b) {
 }
 
 // block-wide sum of fp32 values: float-float (compensated) in and across warps
+template <int NW = kWarps>
 __device__ __forceinline__ FF block_sum_ff(FF v, BlockScratch& s) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v = ff_add(v, ff_shfl_xor(v, o));
@@ -381,10 +439,11 @@ __device__ __forceinline__ FF block_sum_ff(FF v, BlockScratch& s) {
     __syncthreads();
     FF t{s.fred[0], s.fred2[0]};
 #pragma unroll
-    for (int w = 1; w < kWarps; ++w) t = ff_add(t, FF{s.fred[w], s.fred2[w]});
+    for (int w = 1; w < NW; ++w) t = ff_add(t, FF{s.fred[w], s.fred2[w]});
     return t;
 }
-__device__ __forceinline__ FF block_sum_ff(float v, BlockScratch& s) { return block_sum_ff(FF{v, 0.0f}, s); }
+template <int NW = kWarps>
+__device__ __forceinline__ FF block_sum_ff(float v, BlockScratch& s) { return block_sum_ff<NW>(FF{v, 0.0f}, s); }
 
 // ---------------------------------------------------------------------------
 // Block reductions with one barrier each: the warp partials go to one of two
@@ -392,12 +451,13 @@ __device__ __forceinline__ FF block_sum_ff(float v, BlockScratch& s) { return bl
 // ahead into the next reduction never overwrites partials still being read.
 // ---------------------------------------------------------------------------
 struct Red {
-    float f[2][kWarps];
-    float g[2][kWarps];
-    unsigned long long u[2][kWarps];
-    int i[2][kWarps];
+    float f[2][kMaxWarps];
+    float g[2][kMaxWarps];
+    unsigned long long u[2][kMaxWarps];
+    int i[2][kMaxWarps];
 };
 
+template <int NW = kWarps>
 __device__ __forceinline__ float red_max_f32(float v, Red& r, int& par) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
@@ -407,10 +467,11 @@ __device__ __forceinline__ float red_max_f32(float v, Red& r, int& par) {
     __syncthreads();
     float m = buf[0];
 #pragma unroll
-    for (int w = 1; w < kWarps; ++w) m = fmaxf(m, buf[w]);
+    for (int w = 1; w < NW; ++w) m = fmaxf(m, buf[w]);
     return m;
 }
 
+template <int NW = kWarps>
 __device__ __forceinline__ FF red_sum_ff(FF v, Red& r, int& par) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v = ff_add(v, ff_shfl_xor(v, o));
@@ -422,24 +483,32 @@ __device__ __forceinline__ FF red_sum_ff(FF v, Red& r, int& par) {
         bl[threadIdx.x >> 5] = v.lo;
     }
     __syncthreads();
-    FF t{bh[0], bl[0]};
+    // the warp partials combined by a shuffle tree in every warp (log2 NW
+    // dependent steps instead of NW), then taken from lane 0: all threads agree
+    const int lane = threadIdx.x & 31;
+    FF t = lane < NW ? FF{bh[lane], bl[lane]} : FF{0.0f, 0.0f};
 #pragma unroll
-    for (int w = 1; w < kWarps; ++w) t = ff_add(t, FF{bh[w], bl[w]});
-    return t;
+    for (int o = NW / 2; o > 0; o >>= 1) t = ff_add(t, ff_shfl_xor(t, o));
+    return FF{__shfl_sync(0xFFFFFFFFu, t.hi, 0), __shfl_sync(0xFFFFFFFFu, t.lo, 0)};
 }
 
+template <int NW = kWarps>
 __device__ __forceinline__ unsigned long long red_max_u64(unsigned long long v, Red& r, int& par) {
     v = warp_max_u64(v);
     unsigned long long* buf = r.u[par];
     par ^= 1;
     if ((threadIdx.x & 31) == 0) buf[threadIdx.x >> 5] = v;
     __syncthreads();
-    unsigned long long t = 0;
+    unsigned long long t = (threadIdx.x & 31) < NW ? buf[threadIdx.x & 31] : 0ull;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) t = buf[w] > t ? buf[w] : t;
-    return t;
+    for (int o = NW / 2; o > 0; o >>= 1) {
+        const unsigned long long y = __shfl_xor_sync(0xFFFFFFFFu, t, o);
+        t = y > t ? y : t;
+    }
+    return __shfl_sync(0xFFFFFFFFu, t, 0);
 }
 
+template <int NW = kWarps>
 __device__ __forceinline__ int red_sum_int(int v, Red& r, int& par) {
     v = __reduce_add_sync(0xFFFFFFFFu, v);
     int* buf = r.i[par];
@@ -448,11 +517,12 @@ __device__ __forceinline__ int red_sum_int(int v, Red& r, int& par) {
     __syncthreads();
     int t = 0;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) t += buf[w];
+    for (int w = 0; w < NW; ++w) t += buf[w];
     return t;
 }
 
 // exclusive prefix sum in thread order; total in `total`
+template <int NW = kWarps>
 __device__ __forceinline__ int red_scan(int v, int& total, Red& r, int& par) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     int x = v;
@@ -468,7 +538,7 @@ __device__ __forceinline__ int red_scan(int v, int& total, Red& r, int& par) {
     int before = 0;
     total = 0;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) {
+    for (int w = 0; w < NW; ++w) {
         before += (w < warp) ? buf[w] : 0;
         total += buf[w];
     }
@@ -478,18 +548,18 @@ __device__ __forceinline__ int red_scan(int v, int& total, Red& r, int& par) {
 // Partition sum of a block: every thread holds (m, s) = (its maximum, sum of
 // 2^((x - m) c) over its values; m = -inf when it has none).  Returns
 // M = max over the block and the sum rescaled to M as float-float.
+template <int NW = kWarps>
 __device__ __forceinline__ FF red_partition(float m, float s, float c, float& M, Red& r, int& par) {
-    FF v{s, 0.0f};
+    // in the warp: common maximum first, each sum rescaled to it once, then a
+    // plain fp32 tree (5 levels: relative error below 5 * 2^-24)
+    float mw = m;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o);
-        const FF v2 = ff_shfl_xor(v, o);
-        const float mm = fmaxf(m, m2);
-        const FF a = (m == -INFINITY) ? FF{0.0f, 0.0f} : ff_mul(fast_exp2((m - mm) * c), v);
-        const FF b = (m2 == -INFINITY) ? FF{0.0f, 0.0f} : ff_mul(fast_exp2((m2 - mm) * c), v2);
-        v = ff_add(a, b);
-        m = mm;
-    }
+    for (int o = 16; o > 0; o >>= 1) mw = fmaxf(mw, __shfl_xor_sync(0xFFFFFFFFu, mw, o));
+    float sw = (m == -INFINITY) ? 0.0f : s * fast_exp2((m - mw) * c);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sw += __shfl_xor_sync(0xFFFFFFFFu, sw, o);
+    m = mw;
+    FF v{sw, 0.0f};
     float* bm = r.f[par];
     float* bh = r.g[par];
     unsigned long long* bl = r.u[par];
@@ -500,15 +570,23 @@ __device__ __forceinline__ FF red_partition(float m, float s, float c, float& M,
         bl[threadIdx.x >> 5] = (unsigned long long)__float_as_uint(v.lo);
     }
     __syncthreads();
-    M = bm[0];
+    // the same pairwise rescale-and-add over the warp partials, as a shuffle
+    // tree in every warp, taken from lane 0
+    const int lane = threadIdx.x & 31;
+    m = lane < NW ? bm[lane] : -INFINITY;
+    v = lane < NW ? FF{bh[lane], __uint_as_float((uint32_t)bl[lane])} : FF{0.0f, 0.0f};
 #pragma unroll
-    for (int w = 1; w < kWarps; ++w) M = fmaxf(M, bm[w]);
-    FF t{0.0f, 0.0f};
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w)
-        if (bm[w] != -INFINITY)
-            t = ff_add(t, ff_mul(fast_exp2((bm[w] - M) * c), FF{bh[w], __uint_as_float((uint32_t)bl[w])}));
-    return t;
+    for (int o = NW / 2; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o);
+        const FF v2 = ff_shfl_xor(v, o);
+        const float mm = fmaxf(m, m2);
+        const FF a = (m == -INFINITY) ? FF{0.0f, 0.0f} : ff_mul(fast_exp2((m - mm) * c), v);
+        const FF b = (m2 == -INFINITY) ? FF{0.0f, 0.0f} : ff_mul(fast_exp2((m2 - mm) * c), v2);
+        v = ff_add(a, b);
+        m = mm;
+    }
+    M = __shfl_sync(0xFFFFFFFFu, m, 0);
+    return FF{__shfl_sync(0xFFFFFFFFu, v.hi, 0), __shfl_sync(0xFFFFFFFFu, v.lo, 0)};
 }
 
 // exp(l / T - c) for an fp32 logit l and a float-float constant c, to a few
@@ -527,23 +605,22 @@ __device__ __forceinline__ float exp_scaled_minus(float l, float T, FF c) {
 // radix select on 8-bit digits, most significant first: a shared histogram per
 // digit, a block scan over the digits from the top, stop as soon as the keys
 // at or above the current prefix number exactly k.  get(i), i in [0, n)
-// visited as i = tid + j * kThreads, returns a key, or 0 for "no key".
+// visited as i = tid + j * NT (NT threads, NT >= kRadixBins), returns a key, or 0 for "no key".
 // ---------------------------------------------------------------------------
 constexpr int kRadixBins = 256;
-static_assert(kRadixBins == kThreads, "one radix bin per thread");
 
 struct RadixScratch {
-    unsigned long long red_and[kWarps], red_or[kWarps];
-    int wsum[kWarps];
+    unsigned long long red_and[kMaxWarps], red_or[kMaxWarps];
+    int wsum[kMaxWarps];
     int digit, above;
 };
 
-template <class Get>
+template <int NT = kThreads, class Get>
 __device__ unsigned long long block_radix_threshold(Get get, int n, int k, unsigned* hist, RadixScratch& rs) {
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     // common leading bits
     unsigned long long a_and = ~0ull, a_or = 0ull;
-    for (int i = tid; i < n; i += kThreads) {
+    for (int i = tid; i < n; i += NT) {
         const unsigned long long x = get(i);
         if (x) { a_and &= x; a_or |= x; }
     }
@@ -558,7 +635,7 @@ __device__ unsigned long long block_radix_threshold(Get get, int n, int k, unsig
         a_and = ~0ull;
         a_or = 0ull;
 #pragma unroll
-        for (int w = 0; w < kWarps; ++w) { a_and &= rs.red_and[w]; a_or |= rs.red_or[w]; }
+        for (int w = 0; w < NT / 32; ++w) { a_and &= rs.red_and[w]; a_or |= rs.red_or[w]; }
     }
     const unsigned long long diff = a_and ^ a_or;
     if (diff == 0ull) {  // all keys equal
@@ -572,10 +649,10 @@ __device__ unsigned long long block_radix_threshold(Get get, int n, int k, unsig
         const int bits = top >= 8 ? 8 : top;
         const int shift = top - bits;
         const unsigned mask = (1u << bits) - 1u;
-        hist[tid] = 0u;  // kThreads == kRadixBins
+        if (tid < kRadixBins) hist[tid] = 0u;
         if (tid == 0) rs.digit = -1;
         __syncthreads();
-        for (int i = tid; i < n; i += kThreads) {
+        for (int i = tid; i < n; i += NT) {
             const unsigned long long x = get(i);
             if (x == 0ull) continue;
             if (top < 64 && (x >> top) != (prefix >> top)) continue;
@@ -584,7 +661,7 @@ __device__ unsigned long long block_radix_threshold(Get get, int n, int k, unsig
         __syncthreads();
         // thread t owns digit 255 - t (descending order of digits)
         const int d = kRadixBins - 1 - tid;
-        const int h = (int)hist[d];
+        const int h = tid < kRadixBins ? (int)hist[d] : 0;
         int incl = h;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -595,8 +672,8 @@ __device__ unsigned long long block_radix_threshold(Get get, int n, int k, unsig
         __syncthreads();
         int before = above + incl - h;
 #pragma unroll
-        for (int w = 0; w < kWarps; ++w) before += (w < warp) ? rs.wsum[w] : 0;
-        if (before < k && before + h >= k) {
+        for (int w = 0; w < NT / 32; ++w) before += (w < warp) ? rs.wsum[w] : 0;
+        if (h > 0 && before < k && before + h >= k) {
             rs.digit = d;
             rs.above = before;
         }
@@ -664,7 +741,7 @@ __device__ __forceinline__ T warp_kth_largest_of(const T (&x)[N], int k) {
 
 // ---------------------------------------------------------------------------
 // Block-wide k-th largest of n distinct nonzero 64-bit keys (get(i) == 0 means
-// "no key"; i visited as tid + j * kThreads), 1 <= k <= number of keys.  The
+// "no key"; i visited as tid + j * NT, NT >= kRadixBins threads), 1 <= k <= number of keys.  The
 // returned threshold T has exactly k keys >= T.  Rounds over the keys still in
 // play ("live": equal to the prefix found so far above bit `top`): bits common
 // to every live key are taken from their AND at once, the next 8 differing
@@ -673,14 +750,14 @@ __device__ __forceinline__ T warp_kth_largest_of(const T (&x)[N], int k) {
 // class of at most 32 keys is finished by one warp ranking it.
 // ---------------------------------------------------------------------------
 struct SelScratch {
-    unsigned long long red_and[kWarps], red_or[kWarps];
-    int wsum[kWarps];
+    unsigned long long red_and[kMaxWarps], red_or[kMaxWarps];
+    int wsum[kMaxWarps];
     int digit, above, tie_n;
     unsigned long long result;
     unsigned long long tie[32];
 };
 
-template <class Get>
+template <int NT = kThreads, class Get>
 __device__ unsigned long long block_kth_key(Get get, int n, int k, unsigned* hist, SelScratch& ss) {
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     unsigned long long prefix = 0ull;
@@ -692,7 +769,7 @@ __device__ unsigned long long block_kth_key(Get get, int n, int k, unsigned* his
         // common bits of the live keys; the histogram is cleared meanwhile
         unsigned long long a_and = ~0ull, a_or = 0ull;
         int nl = 0;
-        for (int i = tid; i < n; i += kThreads) {
+        for (int i = tid; i < n; i += NT) {
             const unsigned long long x = get(i);
             if (live(x)) {
                 a_and &= x;
@@ -708,14 +785,14 @@ __device__ unsigned long long block_kth_key(Get get, int n, int k, unsigned* his
             ss.red_or[warp] = a_or;
             ss.wsum[warp] = nl;
         }
-        hist[tid] = 0u;  // kThreads == kRadixBins
+        if (tid < kRadixBins) hist[tid] = 0u;
         if (tid == 0) ss.digit = -1;
         __syncthreads();
         a_and = ~0ull;
         a_or = 0ull;
         nl = 0;
 #pragma unroll
-        for (int w = 0; w < kWarps; ++w) {
+        for (int w = 0; w < NT / 32; ++w) {
             a_and &= ss.red_and[w];
             a_or |= ss.red_or[w];
             nl += ss.wsum[w];
@@ -734,14 +811,14 @@ __device__ unsigned long long block_kth_key(Get get, int n, int k, unsigned* his
         const int bits = top >= 8 ? 8 : top;
         const int shift = top - bits;
         const unsigned mask = (1u << bits) - 1u;
-        for (int i = tid; i < n; i += kThreads) {
+        for (int i = tid; i < n; i += NT) {
             const unsigned long long x = get(i);
             if (live(x)) atomicAdd(&hist[(unsigned)(x >> shift) & mask], 1u);
         }
         __syncthreads();
         // thread t owns digit 255 - t: digits in descending order
         const int d = kRadixBins - 1 - tid;
-        const int h = (int)hist[d];
+        const int h = tid < kRadixBins ? (int)hist[d] : 0;
         int incl = h;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -752,7 +829,7 @@ __device__ unsigned long long block_kth_key(Get get, int n, int k, unsigned* his
         __syncthreads();
         int before = above + incl - h;
 #pragma unroll
-        for (int w = 0; w < kWarps; ++w) before += (w < warp) ? ss.wsum[w] : 0;
+        for (int w = 0; w < NT / 32; ++w) before += (w < warp) ? ss.wsum[w] : 0;
         if (h > 0 && before < k && before + h >= k) {
             ss.digit = d;
             ss.above = before;
@@ -773,7 +850,7 @@ __device__ unsigned long long block_kth_key(Get get, int n, int k, unsigned* his
             return prefix;
         }
         if (cnt <= 32) {  // finish the tie class in one warp
-            for (int i = tid; i < n; i += kThreads) {
+            for (int i = tid; i < n; i += NT) {
                 const unsigned long long x = get(i);
                 if (live(x)) ss.tie[atomicAdd(&ss.tie_n, 1)] = x;
             }
@@ -793,6 +870,7 @@ __device__ unsigned long long block_kth_key(Get get, int n, int k, unsigned* his
 }
 
 // exclusive prefix sum over the block (in thread order)
+template <int NW = kWarps>
 __device__ __forceinline__ int block_exclusive_scan(int v, int& total, BlockScratch& s) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     int x = v;
@@ -807,7 +885,7 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int& total, BlockScra
     int before = 0;
     total = 0;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) {
+    for (int w = 0; w < NW; ++w) {
         if (w < warp) before += s.ired[0][w];
         total += s.ired[0][w];
     }

@@ -117,8 +117,7 @@ cudaError_t launch_dependent(void (*kern)(P...), dim3 grid, dim3 block, size_t s
 // aligned: every row starts on a 16-byte boundary, so rows are read with
 // 16-byte vector loads (a row's ragged end element-wise); otherwise element-wise.
 // whole: every CTA's tiles lie in one row (the two halves are streamed side by side)
-cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, bool whole, int grid, size_t smem,
-                          cudaStream_t s);
+cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, int grid, size_t smem, cudaStream_t s);
 cudaError_t launch_prune(const PruneArgs& a, int batch, size_t smem, cudaStream_t s);
 cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid, cudaStream_t s);
 size_t expand_keys_bytes(int max_segments, int support);

@@ -34,7 +34,9 @@ constexpr int kXWarps = kXThreads / 32;
 constexpr int kRegion = 256;    // candidate keys per warp
 constexpr int kVPT = 4;         // 16-byte vectors per thread per tile
 constexpr int kXTileBytes = kVPT * 16 * kXThreads;  // 32 KiB per tile
-constexpr int kStageCap = 32 * kVPT;  // staged vectors per warp: a whole tile's worth
+// staged vectors per warp: flushed once 32 are staged, so a list holding fewer
+// than 32 always has room for a whole tile's worth
+constexpr int kStageCap = 32 + 32 * kVPT;
 // per-warp staging lists while streaming; the bin-ordered list of the top-S sort after
 constexpr int kSpillBytes = kXWarps * kStageCap * (int)(sizeof(uint4) + sizeof(int));
 // two-level histogram of candidate keys: 256 coarse bins (top 8 key bits, two
@@ -607,10 +609,6 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             total += __popc(bal[j]);
         }
         if (total == 0) return;
-        if (scnt + total > kStageCap) {
-            stage_flush<DT>(region, cnt, stage_v, stage_i, scnt, V, theta, S, fine, coarse, &s_theta);
-            scnt = 0;
-        }
 #pragma unroll
         for (int j = 0; j < kVPT; ++j) {
             if ((bal[j] >> lane) & 1u) {
@@ -619,6 +617,11 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
                 stage_i[p] = e0 + (j * kXThreads + tid) * VEC;
             }
             scnt += __popc(bal[j]);
+        }
+        if (scnt >= 32) {  // a full round of one vector per lane
+            __syncwarp();
+            stage_flush<DT>(region, cnt, stage_v, stage_i, scnt, V, theta, S, fine, coarse, &s_theta);
+            scnt = 0;
         }
     };
     // end of the segment of row r that this CTA holds

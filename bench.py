@@ -380,6 +380,27 @@ def main(argv=None):
     ver_ms /= n_k
     assert rheo.status(cfg, ws, stream) == 0
 
+    # tree-attention inputs of the target forward (not part of the tree step):
+    # 20 launches in one graph, averaged over replays
+    attn = rheo.TreeAttn(cfg, device=device)
+    g_attn = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        rheo.tree_attention(cfg, pr, attn, ws, stream)
+        stream.synchronize()
+        with torch.cuda.graph(g_attn, stream=stream):
+            for _ in range(20):
+                rheo.tree_attention(cfg, pr, attn, ws, stream)
+        for _ in range(3):
+            g_attn.replay()
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for _ in range(10):
+            g_attn.replay()
+        a1.record(stream)
+        stream.synchronize()
+    attn_us = a0.elapsed_time(a1) * 1e3 / 200
+    assert rheo.status(cfg, ws, stream) == 0
+
     # end to end through the public API with host buffers: H2D of every input, D2H of the results
     e2e = None
     if rank == 0 or world > 1:
@@ -460,7 +481,9 @@ def main(argv=None):
         "kernels": {"expand_ms_per_step": exp_ms, "expand_ms_by_depth": [x / n_k for x in by_depth],
                     "expand_gbs": exp_gbs, "prune_ms": prune_ms,
                     "verify_ms": ver_ms, "verify_gbs": ver_gbs, "step_gbs": step_gbs,
-                    "step_frac_of_peak": step_gbs / peak},
+                    "step_frac_of_peak": step_gbs / peak,
+                    "tree_attention_us": attn_us,
+                    "tree_attention_bytes": w.batch * (w.budget + 1) * ((w.budget + 1) + 4 + 4 * (w.depth + 1) + 12)},
         "clocks": clocks,
         "gpu_launches": args.steps * (D + 4),  # D expand, 1 prune, 3 verify (prep, stream, residual)
         "e2e": e2e,

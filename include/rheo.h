@@ -170,6 +170,33 @@ int rheo_verify_static(const rheo_config* cfg, const void* target_logits, int64_
                        const rheo_tree* tree, const rheo_pruned* pruned, const rheo_verify_out* out,
                        int32_t* status, rheo_stream_t stream);
 
+/* Inputs of the target forward over the pruned tree (tree attention).  The
+ * paper runs the target model on the tree inside its code base (Sec. 5.1) and
+ * does not define these arrays; the definitions are ours:
+ *   mask      [B, N+1, N+1] uint8: mask[b][i][j] = 1 iff pruned node j is
+ *             node i or an ancestor of i (node i attends to j), else 0;
+ *   position  [B, N+1] int32: depth of pruned node i (root 0); the caller adds
+ *             its context length;
+ *   retrieve  [B, N+1, D+1] int32: row r < n_leaves[b] holds the pruned
+ *             indices of the path from the root to the r-th leaf (leaves =
+ *             nodes without a surviving child, in ascending pruned index),
+ *             position k = the node at depth k, -1 past the leaf's depth;
+ *             rows r >= n_leaves[b] are all -1;
+ *   n_leaves  [B] int32.
+ * Any of the four pointers may be NULL (that output is skipped).  Requires
+ * N+1 <= 4096 (RHEO_EINVAL otherwise).  A pruned tree whose parent of node i
+ * is not in [0, i) (root: -1), or whose depths disagree with its parent
+ * chain, sets RHEO_STATUS_INTERNAL.  The workspace carries the status word. */
+typedef struct {
+    uint8_t* mask;
+    int32_t* position;
+    int32_t* retrieve;
+    int32_t* n_leaves;
+} rheo_tree_attn;
+
+int rheo_tree_attention(const rheo_config* cfg, const rheo_pruned* pruned, const rheo_tree_attn* out,
+                        void* workspace, rheo_stream_t stream);
+
 /* Synchronise the stream, return the device status word in *status (host
  * memory) and clear it.  Returns RHEO_ELAUNCH if the stream reported an error. */
 int rheo_get_status(const rheo_config* cfg, void* workspace, rheo_stream_t stream, int32_t* status);

@@ -99,6 +99,7 @@ def lib():
         L.orc_run_prefix_lm.argtypes = [ctypes.POINTER(_Cfg), _P, _P, ctypes.c_int32,
                                         ctypes.c_int64, ctypes.c_float, ctypes.c_uint64,
                                         ctypes.c_int32, _P, _P]
+        L.orc_tree_attention.argtypes = [ctypes.POINTER(_Cfg), ctypes.POINTER(_Pruned), _P, _P, _P, _P]
     return _lib
 
 
@@ -263,6 +264,26 @@ def verify(cfg: Config, target: np.ndarray, T, seed, offset, tree: Tree, pruned:
     if rc:
         raise OracleError(f"orc_verify returned {rc}")
     return o
+
+
+@dataclass
+class TreeAttention:
+    mask: np.ndarray       # [B, N+1, N+1] uint8
+    position: np.ndarray   # [B, N+1] int32
+    retrieve: np.ndarray   # [B, N+1, D+1] int32
+    n_leaves: np.ndarray   # [B] int32
+
+
+def tree_attention(cfg: Config, pruned: Pruned) -> TreeAttention:
+    """Tree attention inputs of the pruned tree (mask, positions, root-to-leaf paths)."""
+    B, NP, W = cfg.B, cfg.N + 1, cfg.D + 1
+    ta = TreeAttention(np.zeros((B, NP, NP), np.uint8), np.zeros((B, NP), np.int32),
+                       np.zeros((B, NP, W), np.int32), np.zeros(B, np.int32))
+    rc = lib().orc_tree_attention(ctypes.byref(cfg.c()), ctypes.byref(pruned.c()), _ptr(ta.mask),
+                                  _ptr(ta.position), _ptr(ta.retrieve), _ptr(ta.n_leaves))
+    if rc:
+        raise OracleError(f"orc_tree_attention returned {rc}")
+    return ta
 
 
 def philox(ctr, key) -> np.ndarray:

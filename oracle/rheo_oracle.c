@@ -415,6 +415,56 @@ int orc_prune(const orc_cfg* c, const orc_tree* t, orc_pruned* p) {
 }
 
 /* ------------------------------------------------------------------ */
+/* Tree attention inputs for the target forward (our definitions; the  */
+/* paper defers them to its code base, Sec. 5.1)                        */
+/* ------------------------------------------------------------------ */
+
+int orc_tree_attention(const orc_cfg* c, const orc_pruned* p, uint8_t* mask, int32_t* position,
+                       int32_t* retrieve, int32_t* n_leaves) {
+    if (orc_check_cfg(c)) return -1;
+    const int NP = c->N + 1, W = c->D + 1;
+    for (int b = 0; b < c->B; ++b) {
+        const int64_t pb = (int64_t)b * NP;
+        const int32_t* par = p->parent + pb;
+        /* node i attends to itself and to every ancestor: follow the parents */
+        if (mask) {
+            uint8_t* mb = mask + (int64_t)b * NP * NP;
+            memset(mb, 0, (size_t)NP * (size_t)NP);
+            for (int i = 0; i < NP; ++i) {
+                int steps = 0;
+                for (int j = i; j >= 0; j = par[j]) {
+                    if (j >= NP || ++steps > NP) return -3; /* not a tree */
+                    mb[(int64_t)i * NP + j] = 1;
+                }
+            }
+        }
+        if (position)
+            for (int i = 0; i < NP; ++i) position[pb + i] = p->depth[pb + i];
+        /* leaves in ascending pruned index; the path of each, root first */
+        int nl = 0;
+        if (retrieve)
+            for (int64_t q = 0; q < (int64_t)NP * W; ++q) retrieve[pb * W + q] = -1;
+        for (int i = 0; i < NP; ++i) {
+            if (p->n_child[pb + i] != 0) continue;
+            if (retrieve) {
+                const int dep = p->depth[pb + i];
+                if (dep < 0 || dep >= W) return -3;
+                int k = dep;
+                for (int j = i; j >= 0; j = par[j]) {
+                    if (k < 0) return -3; /* depth disagrees with the parent chain */
+                    retrieve[(pb + nl) * W + k] = j;
+                    --k;
+                }
+                if (k != -1) return -3;
+            }
+            ++nl;
+        }
+        if (n_leaves) n_leaves[b] = nl;
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
 /* RheoVerification, layer by layer (Algorithm 1, Theorem 1)            */
 /* ------------------------------------------------------------------ */
 

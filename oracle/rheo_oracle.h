@@ -108,6 +108,19 @@ int orc_run_prefix_lm(const orc_cfg* c, const float* draft_table, const float* t
                       int32_t table_depth, int64_t n_trials, float T, uint64_t seed0, int32_t L,
                       int32_t* streams, int32_t* acc_len);
 
+/* Inputs of the target forward over the pruned tree (tree attention).  The
+ * paper leaves them to its code base (Sec. 5.1); the definitions are ours:
+ *   mask[b][i][j] = 1 iff pruned node j is node i or an ancestor of i, else 0
+ *                   ([B][N+1][N+1] bytes);
+ *   position[b][i] = depth of pruned node i (root 0);
+ *   leaves = pruned nodes without a surviving child, in ascending pruned index;
+ *   retrieve[b][r][k] = pruned index of the depth-k node on the path from the
+ *                   root to the r-th leaf ([B][N+1][D+1]), -1 past the leaf's
+ *                   depth and on every row r >= n_leaves[b].
+ * Computed by following parent pointers.  Any output may be NULL. */
+int orc_tree_attention(const orc_cfg* c, const orc_pruned* p, uint8_t* mask, int32_t* position,
+                       int32_t* retrieve, int32_t* n_leaves);
+
 #ifdef __cplusplus
 }
 #endif

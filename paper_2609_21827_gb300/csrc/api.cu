@@ -216,6 +216,26 @@ extern "C" int rheo_prune(const rheo_config* cfg, const rheo_tree* tree, const r
     return launch_prune(a, cfg->batch, smem, (cudaStream_t)stream) == cudaSuccess ? RHEO_OK : RHEO_ELAUNCH;
 }
 
+extern "C" int rheo_tree_attention(const rheo_config* cfg, const rheo_pruned* pruned, const rheo_tree_attn* out,
+                                   void* ws, rheo_stream_t stream) {
+    if (!valid(cfg) || !pruned || !pruned->parent || !pruned->depth || !pruned->n_child || !out || !ws ||
+        cfg->budget + 1 > 4096)
+        return RHEO_EINVAL;
+    if (!out->mask && !out->position && !out->retrieve && !out->n_leaves) return RHEO_OK;
+    const Layout L = layout(*cfg);
+    TreeAttnArgs a;
+    a.n = dims(*cfg);
+    a.pr = pruned_ptrs(pruned);
+    a.mask = out->mask;
+    a.position = out->position;
+    a.retrieve = out->retrieve;
+    a.n_leaves = out->n_leaves;
+    a.status = at<unsigned>(ws, L.status);
+    return launch_tree_attn(a, cfg->batch, tree_attn_smem_bytes(cfg->budget), (cudaStream_t)stream) == cudaSuccess
+               ? RHEO_OK
+               : RHEO_ELAUNCH;
+}
+
 extern "C" int rheo_verify(const rheo_config* cfg, const void* logits, int64_t row_stride, const float* temperature,
                            const uint64_t* seed, const uint64_t* offset, const rheo_tree* tree,
                            const rheo_pruned* pruned, const rheo_verify_out* out, void* ws, rheo_stream_t stream) {

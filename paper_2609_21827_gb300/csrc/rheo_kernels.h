@@ -63,6 +63,16 @@ struct PruneArgs {
     unsigned* status;
 };
 
+struct TreeAttnArgs {
+    Dims n;
+    PrunedPtrs pr;
+    uint8_t* mask;       // [B, N+1, N+1] or null
+    int32_t* position;   // [B, N+1] or null
+    int32_t* retrieve;   // [B, N+1, D+1] or null
+    int32_t* n_leaves;   // [B] or null
+    unsigned* status;
+};
+
 struct VerifyArgs {
     Dims n;                         // n.chunks: 2 KB chunks per target row
     int units;                      // warps of the stream launch with work (one contiguous run of chunks each)
@@ -123,6 +133,8 @@ cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid
 size_t expand_keys_bytes(int max_segments, int support);
 size_t expand_smem_bytes(int max_segments, int support);
 int expand_tile_elems(int dtype);
+cudaError_t launch_tree_attn(const TreeAttnArgs& a, int batch, size_t smem, cudaStream_t s);
+size_t tree_attn_smem_bytes(int budget);
 int verify_table_width(int K);
 int verify_chunks_per_row(int dtype, int V);
 int verify_stream_grid(int sms, int64_t chunks);

@@ -20,6 +20,7 @@ STATUS_BAD_LOGIT, STATUS_EMPTY_ROW, STATUS_BAD_TEMPERATURE, STATUS_INTERNAL = 1,
 SLOT_ROOT, SLOT_LEAD, SLOT_SAMPLED, SLOT_FILL = 0, 1, 2, 3
 
 EXPORTS = ("rheo_sizes", "rheo_workspace_init", "rheo_expand", "rheo_prune", "rheo_verify", "rheo_verify_static",
+           "rheo_tree_attention",
            "rheo_get_status")
 
 
@@ -51,6 +52,10 @@ class _VerifyOut(ctypes.Structure):
                                    "row_lse")]
 
 
+class _TreeAttn(ctypes.Structure):
+    _fields_ = [(n, _VP) for n in ("mask", "position", "retrieve", "n_leaves")]
+
+
 _lib = None
 
 
@@ -77,6 +82,7 @@ def lib():
         L.rheo_verify_static.argtypes = [C, _VP, ctypes.c_int64, _VP, _VP, _VP, ctypes.POINTER(_Tree),
                                          ctypes.POINTER(_Pruned), ctypes.POINTER(_VerifyOut), _VP, _VP]
         L.rheo_get_status.argtypes = [C, _VP, _VP, ctypes.POINTER(ctypes.c_int32)]
+        L.rheo_tree_attention.argtypes = [C, ctypes.POINTER(_Pruned), ctypes.POINTER(_TreeAttn), _VP, _VP]
         for name in EXPORTS:
             getattr(L, name).restype = ctypes.c_int
         _lib = L
@@ -234,6 +240,25 @@ def expand(cfg: Config, d: int, logits: torch.Tensor, temperature: torch.Tensor,
 def prune(cfg: Config, tree: Tree, pruned: Pruned, ws: Workspace, stream=None) -> None:
     _check(lib().rheo_prune(ctypes.byref(cfg.c()), ctypes.byref(tree.c()), ctypes.byref(pruned.c()), ws.ptr(),
                             _stream(stream)), "rheo_prune")
+
+
+class TreeAttn:
+    """Outputs of rheo_tree_attention (ancestor mask, positions, root-to-leaf paths)."""
+
+    def __init__(self, cfg: Config, device="cuda"):
+        B, NP, W = cfg.batch, cfg.budget + 1, cfg.depth + 1
+        self.mask = torch.zeros((B, NP, NP), dtype=torch.uint8, device=device)
+        self.position = torch.zeros((B, NP), dtype=torch.int32, device=device)
+        self.retrieve = torch.zeros((B, NP, W), dtype=torch.int32, device=device)
+        self.n_leaves = torch.zeros((B,), dtype=torch.int32, device=device)
+
+    def c(self) -> _TreeAttn:
+        return _TreeAttn(*[getattr(self, n).data_ptr() for n, _ in _TreeAttn._fields_])
+
+
+def tree_attention(cfg: Config, pruned: Pruned, out: TreeAttn, ws: Workspace, stream=None) -> None:
+    _check(lib().rheo_tree_attention(ctypes.byref(cfg.c()), ctypes.byref(pruned.c()), ctypes.byref(out.c()),
+                                     ws.ptr(), _stream(stream)), "rheo_tree_attention")
 
 
 def verify(cfg: Config, logits: torch.Tensor, temperature: torch.Tensor, seed: torch.Tensor,

@@ -188,18 +188,22 @@ def oracle_cycle_seconds(w, draft, reqs):
 
 
 def cpu_baseline(w, draft, budget_s=15.0):
-    """The oracle as it stands, on the host cores, over a bounded sample of requests."""
+    """The oracle as it stands, on the host cores, over a bounded sample: whole
+    cycles of the batch (or of its first requests) repeated for about budget_s."""
     import oracle
 
     oracle.build()
     cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
     first = oracle_cycle_seconds(w, draft, [0])
     n = max(1, min(w.batch, int(budget_s / max(first, 1e-3))))
-    secs = oracle_cycle_seconds(w, draft, range(n)) if n > 1 else first
-    per_step = secs * w.batch / n
+    secs, cycles = 0.0, 0
+    while cycles == 0 or (secs < budget_s * 0.7 and cycles < 50):
+        secs += oracle_cycle_seconds(w, draft, range(n)) if n > 1 else first
+        cycles += 1
+    per_step = secs / cycles * w.batch / n
     return {"value": 1.0 / per_step, "unit": "tree-steps/s", "cores": min(cores, max(n, w.K)),
             "kind": "oracle",
-            "sample": f"{n} of {w.batch} requests of one {w.name} cycle ({secs:.1f} s), scaled to the full batch"}
+            "sample": f"{cycles} cycles of {n} of {w.batch} requests of {w.name} ({secs:.1f} s), scaled to the full batch"}
 
 
 def build_inputs(w, device):
@@ -401,6 +405,46 @@ def main(argv=None):
     attn_us = a0.elapsed_time(a1) * 1e3 / 200
     assert rheo.status(cfg, ws, stream) == 0
 
+    # verification variants (App. A, App. D.2) on the same trees and targets:
+    # per-call time on this step's tree, and the mean accepted length over the
+    # requests of 8 more cycles (Philox offsets 1..8), paired across variants
+    variants = {}
+    names = {"rheo": rheo.VERIFY_RHEO, "rrsw": rheo.VERIFY_RRSW, "onehot": rheo.VERIFY_ONEHOT}
+    vout = rheo.VerifyOut(cfg, row_lse=False, device=device)
+    for name, v in names.items():
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                rheo.verify_variant(cfg, v, target, draft.temperature, draft.seed, draft.offset, tree, pr, vout, ws,
+                                    stream)
+            v0, v1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            v0.record(stream)
+            for _ in range(50):
+                rheo.verify_variant(cfg, v, target, draft.temperature, draft.seed, draft.offset, tree, pr, vout, ws,
+                                    stream)
+            v1.record(stream)
+            stream.synchronize()
+        variants[name] = {"verify_us": v0.elapsed_time(v1) * 1e3 / 50, "accepted": []}
+    off0 = draft.offset.clone()
+    for off in range(1, 9):
+        draft.offset.fill_(off)
+        tr2, pr2 = rheo.Tree(cfg, device=device), rheo.Pruned(cfg, device=device)
+        fr2 = []
+        for d in range(1, D + 1):
+            rheo.expand(cfg, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tr2, ws)
+            if d < D:
+                fr2.append(tr2.frontier.clone())
+        rheo.prune(cfg, tr2, pr2, ws)
+        tg2 = synth.target_rows(w, draft, fr2, pr2.gen_id)
+        for name, v in names.items():
+            rheo.verify_variant(cfg, v, tg2, draft.temperature, draft.seed, draft.offset, tr2, pr2, vout, ws)
+            variants[name]["accepted"] += vout.accepted_len.cpu().tolist()
+    draft.offset.copy_(off0)
+    assert rheo.status(cfg, ws) == 0
+    for name in names:
+        acc = variants[name].pop("accepted")
+        variants[name]["mean_accepted"] = sum(acc) / len(acc)
+        variants[name]["samples"] = len(acc)
+
     # end to end through the public API with host buffers: H2D of every input, D2H of the results
     e2e = None
     if rank == 0 or world > 1:
@@ -483,6 +527,7 @@ def main(argv=None):
                     "verify_ms": ver_ms, "verify_gbs": ver_gbs, "step_gbs": step_gbs,
                     "step_frac_of_peak": step_gbs / peak,
                     "tree_attention_us": attn_us,
+                    "verify_variants": variants,
                     "tree_attention_bytes": w.batch * (w.budget + 1) * ((w.budget + 1) + 4 + 4 * (w.depth + 1) + 12)},
         "clocks": clocks,
         "gpu_launches": args.steps * (D + 4),  # D expand, 1 prune, 3 verify (prep, stream, residual)

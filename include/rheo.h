@@ -152,6 +152,30 @@ int rheo_verify(const rheo_config* cfg, const void* target_logits, int64_t row_s
                 const rheo_tree* tree, const rheo_pruned* pruned, const rheo_verify_out* out,
                 void* workspace, rheo_stream_t stream);
 
+/* Verification variants on the same kernels (App. A, App. D.2), for
+ * comparisons of acceptance; all are lossless.  variant:
+ *   RHEO_VERIFY_RHEO    Algorithm 1 (exactly rheo_verify);
+ *   RHEO_VERIFY_RRSW    recursive rejection without replacement (App. D.2):
+ *                       leads (slots < m) one-hot against p in slot order;
+ *                       then the sampled child against the renormalised
+ *                       residual p~ = r/M: accept iff fp32(eta*q~)*M <= r(Y);
+ *                       on rejection the tail residual becomes max(0, r - M q~)
+ *                       (mass M - sum_tail min(r, M q~)); then the fills
+ *                       (slots > m) one-hot against it;
+ *   RHEO_VERIFY_ONEHOT  vanilla verification of the pool as a top-K set
+ *                       (Sec. 2.2, App. A): every surviving child, the sampled
+ *                       one too, one-hot against r = p in slot order.
+ * One-hot test of child c: accept iff eta*M <= r(c), else M -= r(c), r(c) = 0.
+ * Coins: tag 2, draw 0 for the sampled child's test under RRSW, draw 1+slot for
+ * every one-hot test.  The final draw after all rejections is u* ~ r over V
+ * minus the surviving children, as in rheo_verify.  Other arguments, outputs
+ * and errors as rheo_verify; an unknown variant returns RHEO_EINVAL. */
+enum { RHEO_VERIFY_RHEO = 0, RHEO_VERIFY_RRSW = 1, RHEO_VERIFY_ONEHOT = 2 };
+int rheo_verify_variant(const rheo_config* cfg, int32_t variant, const void* target_logits, int64_t row_stride,
+                        const float* temperature, const uint64_t* seed, const uint64_t* offset,
+                        const rheo_tree* tree, const rheo_pruned* pruned, const rheo_verify_out* out,
+                        void* workspace, rheo_stream_t stream);
+
 /* Verification for callers that cannot allocate device memory where they
  * verify (code handed only fixed input/output buffers by a host framework,
  * runtimes whose device memory is partitioned up front, loops that must not

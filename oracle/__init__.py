@@ -42,12 +42,16 @@ def build(force: bool = False) -> str:
     return _SO
 
 
+VERIFY_RHEO, VERIFY_RRSW, VERIFY_ONEHOT = 0, 1, 2
+
+
 class _Cfg(ctypes.Structure):
     _fields_ = [
         ("B", ctypes.c_int32), ("V", ctypes.c_int32), ("K", ctypes.c_int32),
         ("m", ctypes.c_int32), ("S", ctypes.c_int32), ("D", ctypes.c_int32),
         ("N", ctypes.c_int32), ("eps", ctypes.c_double),
         ("proxy_mode", ctypes.c_int32), ("fixed_log_proxy", ctypes.c_double),
+        ("verify_mode", ctypes.c_int32),
     ]
 
 
@@ -122,6 +126,7 @@ class Config:
     eps: float = 1e-6
     proxy_mode: int = 0
     fixed_log_proxy: float = 0.0
+    verify_mode: int = 0  # VERIFY_RHEO, VERIFY_RRSW or VERIFY_ONEHOT
 
     def __post_init__(self):
         if self.S is None:
@@ -129,7 +134,7 @@ class Config:
 
     def c(self) -> _Cfg:
         return _Cfg(self.B, self.V, self.K, self.m, self.S, self.D, self.N, self.eps,
-                    self.proxy_mode, self.fixed_log_proxy)
+                    self.proxy_mode, self.fixed_log_proxy, self.verify_mode)
 
     @property
     def G1(self) -> int:

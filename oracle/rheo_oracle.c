@@ -58,6 +58,7 @@ int orc_check_cfg(const orc_cfg* c) {
     if (G1 > ORC_MAX_NODES) return -1;
     if (c->N < 1 || c->N > G1 - 1) return -1;
     if (c->m == 0 && !(c->eps > 0.0)) return -1;
+    if (c->verify_mode < ORC_VERIFY_RHEO || c->verify_mode > ORC_VERIFY_ONEHOT) return -1;
     return 0;
 }
 
@@ -468,6 +469,87 @@ int orc_tree_attention(const orc_cfg* c, const orc_pruned* p, uint8_t* mask, int
 /* RheoVerification, layer by layer (Algorithm 1, Theorem 1)            */
 /* ------------------------------------------------------------------ */
 
+/* The verification variants at one node u (target row l, log-partition lu):
+ * returns the accepted pruned index or -1, and leaves the residual mass in *M,
+ * and, when the sampled child was rejected, the tail residual in rhat (indexed
+ * through tail_pos) with *use_tail = 1.  The rules are those of orc_cfg's
+ * verify_mode.  Coins: draw 0 for the sampled child under RRSW, draw 1+slot
+ * for every one-hot candidate (the sampled child too under ONEHOT). */
+static int verify_variant(const orc_cfg* c, int b, const float* l, double lu, float T, uint64_t seed,
+                          uint64_t offset, const orc_tree* t, const orc_pruned* p, int u, double* gap_out,
+                          float* rhat, int32_t* tail_pos, const int32_t** tids_out, double* M_out,
+                          int* use_tail_out) {
+    const int N = c->N, TL = c->S - c->m;
+    const int64_t G1 = orc_nodes_per_request(c), E = orc_expansions_per_request(c);
+    const int64_t nb = (int64_t)b * G1, pb = (int64_t)b * (N + 1);
+    const int fc = p->first_child[pb + u], nc = p->n_child[pb + u], sc = p->sampled_child[pb + u];
+    const int64_t gu = p->gen_id[pb + u];
+    double M = 1.0;
+    int use_tail = 0;
+#define P_OF(tok) ((float)exp((double)l[(tok)] / (double)T - lu))
+    /* one-hot rejection of child v against the current residual (mass M) */
+#define ONE_HOT(v)                                                                                        \
+    do {                                                                                                  \
+        const int64_t gv_ = p->gen_id[pb + (v)];                                                         \
+        const int tok_ = p->token[pb + (v)];                                                             \
+        const float eta_ = orc_uniform(seed, offset, ORC_TAG_VERIFY, (int32_t)gu,                        \
+                                       (uint64_t)(1 + slot_of(c, gv_)));                                 \
+        float rv_;                                                                                       \
+        if (use_tail && tail_pos[tok_] >= 0) rv_ = rhat[tail_pos[tok_]];                                 \
+        else rv_ = P_OF(tok_);                                                                           \
+        const double lhs_ = (double)eta_ * M;                                                            \
+        const double gap_ = rel_gap(lhs_, rv_);                                                          \
+        if (gap_ < *gap_out) *gap_out = gap_;                                                            \
+        if (lhs_ <= (double)rv_) { accepted = (v); goto done; }                                          \
+        M -= (double)rv_;                                                                                \
+        if (use_tail && tail_pos[tok_] >= 0) rhat[tail_pos[tok_]] = 0.0f;                                \
+    } while (0)
+    int accepted = -1;
+    if (c->verify_mode == ORC_VERIFY_ONEHOT) {
+        for (int k = 0; k < nc; ++k) ONE_HOT(fc + k);
+        goto done;
+    }
+    /* RRSw: the leads under p */
+    for (int k = 0; k < nc; ++k)
+        if (t->slot[nb + p->gen_id[pb + fc + k]] == ORC_SLOT_LEAD) ONE_HOT(fc + k);
+    if (sc >= 0) {
+        /* the sampled child against p~ = r / M: accept iff eta*q~ <= r(Y) / M */
+        const int64_t gs = p->gen_id[pb + sc];
+        const float eta0 = orc_uniform(seed, offset, ORC_TAG_VERIFY, (int32_t)gu, 0);
+        const float qv = t->qtilde[nb + gs];
+        const float pv = P_OF(p->token[pb + sc]);
+        const double lhs = (double)(eta0 * qv) * M; /* fp32(eta*q~), then times M */
+        const double gap = rel_gap(lhs, pv);
+        if (gap < *gap_out) *gap_out = gap;
+        if (lhs <= (double)pv) { accepted = sc; goto done; }
+        /* residual M * norm(max(0, p~ - q~)) = max(0, r - M q~) on the tail */
+        const int64_t e = parent_expansion_of(c, gs);
+        const int32_t* tids = t->tail_ids + ((int64_t)b * E + e) * TL;
+        const float* tq = t->tail_q + ((int64_t)b * E + e) * TL;
+        double overlap = 0.0;
+        for (int i = 0; i < TL; ++i) {
+            const float pt = P_OF(tids[i]);
+            const double mq = M * (double)tq[i];
+            const double d = (double)pt - mq;
+            rhat[i] = d > 0.0 ? (float)d : 0.0f;
+            overlap += (double)pt < mq ? (double)pt : mq;
+            tail_pos[tids[i]] = i;
+        }
+        M -= overlap;
+        use_tail = 1;
+        *tids_out = tids;
+    }
+    /* the fills against the residual */
+    for (int k = 0; k < nc; ++k)
+        if (t->slot[nb + p->gen_id[pb + fc + k]] == ORC_SLOT_FILL) ONE_HOT(fc + k);
+done:
+#undef ONE_HOT
+#undef P_OF
+    *M_out = M;
+    *use_tail_out = use_tail;
+    return accepted;
+}
+
 static int verify_request(const orc_cfg* c, int b, const float* target, float T, uint64_t seed,
                           uint64_t offset, const orc_tree* t, const orc_pruned* p, orc_verify_out* o) {
     const int V = c->V, N = c->N, D = c->D, K = c->K, TL = c->S - c->m;
@@ -512,51 +594,56 @@ static int verify_request(const orc_cfg* c, int b, const float* target, float T,
         int use_tail = 0;
         const int32_t* tids = NULL;
         int accepted = -1;
-        if (nc > 0 && sc >= 0) {
-            /* stochastic-first: accept u_s with probability min(1, p/q~) */
-            const int64_t gs = p->gen_id[pb + sc];
-            const float eta0 = orc_uniform(seed, offset, ORC_TAG_VERIFY, (int32_t)gu, 0);
-            const float qv = t->qtilde[nb + gs];
-            const float pv = P_OF(p->token[pb + sc]);
-            const float lhs = eta0 * qv; /* fp32 */
-            double gap = rel_gap(lhs, pv);
-            if (gap < gl[len]) gl[len] = gap;
-            if (lhs <= pv) {
-                accepted = sc;
-            } else {
-                /* residual r = norm(max(0, p - q~)), kept unnormalised with mass M */
-                const int64_t e = parent_expansion_of(c, gs);
-                tids = t->tail_ids + ((int64_t)b * E + e) * TL;
-                const float* tq = t->tail_q + ((int64_t)b * E + e) * TL;
-                double overlap = 0.0;
-                for (int i = 0; i < TL; ++i) {
-                    float pt = P_OF(tids[i]);
-                    rhat[i] = pt - tq[i] > 0.0f ? pt - tq[i] : 0.0f;
-                    overlap += (double)(pt < tq[i] ? pt : tq[i]);
-                    tail_pos[tids[i]] = i;
-                }
-                M = 1.0 - overlap;
-                use_tail = 1;
-            }
-        }
-        if (accepted < 0 && nc > 0) {
-            /* recursive rejection over the remaining candidates in slot order */
-            for (int k = 0; k < nc; ++k) {
-                const int v = fc + k;
-                if (v == sc) continue;
-                const int64_t gv = p->gen_id[pb + v];
-                const int tok = p->token[pb + v];
-                const float eta = orc_uniform(seed, offset, ORC_TAG_VERIFY, (int32_t)gu,
-                                              (uint64_t)(1 + slot_of(c, gv)));
-                float rv;
-                if (use_tail && tail_pos[tok] >= 0) rv = rhat[tail_pos[tok]];
-                else rv = P_OF(tok);
-                const double lhs = (double)eta * M;
-                double gap = rel_gap(lhs, rv);
+        if (c->verify_mode != ORC_VERIFY_RHEO) {
+            accepted = verify_variant(c, b, l, lu, T, seed, offset, t, p, u, gl + len, rhat, tail_pos, &tids,
+                                      &M, &use_tail);
+        } else {
+            if (nc > 0 && sc >= 0) {
+                /* stochastic-first: accept u_s with probability min(1, p/q~) */
+                const int64_t gs = p->gen_id[pb + sc];
+                const float eta0 = orc_uniform(seed, offset, ORC_TAG_VERIFY, (int32_t)gu, 0);
+                const float qv = t->qtilde[nb + gs];
+                const float pv = P_OF(p->token[pb + sc]);
+                const float lhs = eta0 * qv; /* fp32 */
+                double gap = rel_gap(lhs, pv);
                 if (gap < gl[len]) gl[len] = gap;
-                if (lhs <= (double)rv) { accepted = v; break; }
-                M -= (double)rv;
-                if (use_tail && tail_pos[tok] >= 0) rhat[tail_pos[tok]] = 0.0f;
+                if (lhs <= pv) {
+                    accepted = sc;
+                } else {
+                    /* residual r = norm(max(0, p - q~)), kept unnormalised with mass M */
+                    const int64_t e = parent_expansion_of(c, gs);
+                    tids = t->tail_ids + ((int64_t)b * E + e) * TL;
+                    const float* tq = t->tail_q + ((int64_t)b * E + e) * TL;
+                    double overlap = 0.0;
+                    for (int i = 0; i < TL; ++i) {
+                        float pt = P_OF(tids[i]);
+                        rhat[i] = pt - tq[i] > 0.0f ? pt - tq[i] : 0.0f;
+                        overlap += (double)(pt < tq[i] ? pt : tq[i]);
+                        tail_pos[tids[i]] = i;
+                    }
+                    M = 1.0 - overlap;
+                    use_tail = 1;
+                }
+            }
+            if (accepted < 0 && nc > 0) {
+                /* recursive rejection over the remaining candidates in slot order */
+                for (int k = 0; k < nc; ++k) {
+                    const int v = fc + k;
+                    if (v == sc) continue;
+                    const int64_t gv = p->gen_id[pb + v];
+                    const int tok = p->token[pb + v];
+                    const float eta = orc_uniform(seed, offset, ORC_TAG_VERIFY, (int32_t)gu,
+                                                  (uint64_t)(1 + slot_of(c, gv)));
+                    float rv;
+                    if (use_tail && tail_pos[tok] >= 0) rv = rhat[tail_pos[tok]];
+                    else rv = P_OF(tok);
+                    const double lhs = (double)eta * M;
+                    double gap = rel_gap(lhs, rv);
+                    if (gap < gl[len]) gl[len] = gap;
+                    if (lhs <= (double)rv) { accepted = v; break; }
+                    M -= (double)rv;
+                    if (use_tail && tail_pos[tok] >= 0) rhat[tail_pos[tok]] = 0.0f;
+                }
             }
         }
         if (accepted >= 0) {

@@ -45,7 +45,19 @@ typedef struct {
     double eps;      /* proxy offset for m = 0 */
     int32_t proxy_mode;      /* 0: the paper's proxy. 1: fixed log-proxy (planted mistake for tests) */
     double fixed_log_proxy;  /* used only when proxy_mode == 1 */
+    int32_t verify_mode;     /* ORC_VERIFY_*: the verification rule applied at every node */
 } orc_cfg;
+
+/* Verification rules (all lossless):
+ *  RHEO    Algorithm 1: the sampled child first (accept iff eta*q~ <= p), then
+ *          the others in slot order against r = norm(max(0, p - q~));
+ *  RRSW    recursive rejection, App. D.2: the leads in slot order by one-hot
+ *          rejection under p, then the sampled child against the renormalised
+ *          residual p~ (accept iff eta*q~ <= p~), then the fills against
+ *          norm(max(0, p~ - q~));
+ *  ONEHOT  vanilla verification of a top-K tree (Sec. 2.2, App. A): every child
+ *          a one-hot candidate in slot order, residual from p. */
+enum { ORC_VERIFY_RHEO = 0, ORC_VERIFY_RRSW = 1, ORC_VERIFY_ONEHOT = 2 };
 
 typedef struct {
     int32_t* token;      /* [B*G1] token of each generated node; root -1 */

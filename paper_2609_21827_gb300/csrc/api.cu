@@ -236,9 +236,11 @@ extern "C" int rheo_tree_attention(const rheo_config* cfg, const rheo_pruned* pr
                : RHEO_ELAUNCH;
 }
 
-extern "C" int rheo_verify(const rheo_config* cfg, const void* logits, int64_t row_stride, const float* temperature,
-                           const uint64_t* seed, const uint64_t* offset, const rheo_tree* tree,
-                           const rheo_pruned* pruned, const rheo_verify_out* out, void* ws, rheo_stream_t stream) {
+extern "C" int rheo_verify_variant(const rheo_config* cfg, int32_t variant, const void* logits, int64_t row_stride,
+                                   const float* temperature, const uint64_t* seed, const uint64_t* offset,
+                                   const rheo_tree* tree, const rheo_pruned* pruned, const rheo_verify_out* out,
+                                   void* ws, rheo_stream_t stream) {
+    if (variant != RHEO_VERIFY_RHEO && variant != RHEO_VERIFY_RRSW && variant != RHEO_VERIFY_ONEHOT) return RHEO_EINVAL;
     if (!valid(cfg) || !logits || row_stride < cfg->vocab || !temperature || !seed || !offset || !tree_ok(tree) ||
         !pruned_ok(pruned) || !out || !out->accepted_len || !out->accepted_tokens || !out->accepted_nodes ||
         !out->bonus_token || !ws)
@@ -246,6 +248,7 @@ extern "C" int rheo_verify(const rheo_config* cfg, const void* logits, int64_t r
     const Layout L = layout(*cfg);
     VerifyArgs a;
     a.n = dims(*cfg);
+    a.variant = variant == RHEO_VERIFY_RRSW ? kVerifyRrsw : variant == RHEO_VERIFY_ONEHOT ? kVerifyOneHot : kVerifyRheo;
     a.logits = static_cast<const char*>(logits);
     a.row_stride_bytes = row_stride * elem_size(*cfg);
     a.T = temperature;
@@ -282,6 +285,13 @@ extern "C" int rheo_verify(const rheo_config* cfg, const void* logits, int64_t r
                    cudaSuccess
                ? RHEO_OK
                : RHEO_ELAUNCH;
+}
+
+extern "C" int rheo_verify(const rheo_config* cfg, const void* logits, int64_t row_stride, const float* temperature,
+                           const uint64_t* seed, const uint64_t* offset, const rheo_tree* tree,
+                           const rheo_pruned* pruned, const rheo_verify_out* out, void* ws, rheo_stream_t stream) {
+    return rheo_verify_variant(cfg, RHEO_VERIFY_RHEO, logits, row_stride, temperature, seed, offset, tree, pruned, out,
+                               ws, stream);
 }
 
 extern "C" int rheo_get_status(const rheo_config* cfg, void* ws, rheo_stream_t stream, int32_t* status) {

@@ -73,8 +73,11 @@ struct TreeAttnArgs {
     unsigned* status;
 };
 
+enum : int { kVerifyRheo = 0, kVerifyRrsw = 1, kVerifyOneHot = 2 };
+
 struct VerifyArgs {
     Dims n;                         // n.chunks: 2 KB chunks per target row
+    int variant = kVerifyRheo;      // verification rule at every node (kVerify*)
     int units;                      // warps of the stream launch with work (one contiguous run of chunks each)
     const char* logits;
     int64_t row_stride_bytes;

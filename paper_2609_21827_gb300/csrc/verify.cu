@@ -231,6 +231,103 @@ __device__ __forceinline__ float exp_ff_minus(FF x, FF c) {
 
 // The decision table of pruned row r (Algorithm 1 at the node), built by one
 // warp from the row's segment partials and its record.
+// Vanilla verification of the node's children as a top-K pool (Sec. 2.2,
+// App. A): every surviving child, the sampled one too, a one-hot candidate in
+// slot order against r^ = p; coin draw 1+slot.  Lane 0.
+__device__ void onehot_walk(const WarpRow& w, int nc, int fc, float* tab) {
+    FF M{1.0f, 0.0f};
+    int acc = -1;
+    for (int c2 = 0; c2 < nc; ++c2) {
+        const float eta = w.coin[1 + w.tok[c2]];
+        if (ff_le(ff_mul(eta, M), w.pc[c2])) {
+            acc = fc + c2;
+            break;
+        }
+        M = ff_add(M, -w.pc[c2]);
+    }
+    tab[0] = 1.0f;
+    tab[1] = 0.0f;
+    tab[5] = 0.0f;
+    tab[6] = (float)acc;
+}
+
+// Recursive rejection without replacement on the hybrid pool (App. D.2): the
+// leads (slots < m) one-hot against p, then the sampled child against the
+// renormalised residual p~ = r^ / M (accept iff fp32(eta q~) * M <= p), then on
+// its rejection the tail residual becomes max(0, r^ - M q~) and the fills
+// (slots > m) go one-hot against it.  Whole warp (the tail is spread over the
+// lanes); coins: draw 0 for the sampled child, draw 1+slot otherwise.
+__device__ void rrsw_walk(const VerifyArgs& a, int64_t r, WarpRow& w, int nc, int fc, int sc, float qs,
+                          const int (&cpos)[4], const float (&tq)[4], const FF (&tx)[4], FF lse, float* tab) {
+    const int lane = threadIdx.x & 31;
+    const int m = a.n.m, TL = a.n.TL;
+    FF M{1.0f, 0.0f};
+    int acc = -1;
+    if (lane == 0)
+        for (int c2 = 0; c2 < nc; ++c2) {
+            if (w.tok[c2] >= m) continue;  // leads only
+            const float eta = w.coin[1 + w.tok[c2]];
+            if (ff_le(ff_mul(eta, M), w.pc[c2])) {
+                acc = fc + c2;
+                break;
+            }
+            M = ff_add(M, -w.pc[c2]);
+        }
+    acc = __shfl_sync(0xFFFFFFFFu, acc, 0);
+    M = FF{__shfl_sync(0xFFFFFFFFu, M.hi, 0), __shfl_sync(0xFFFFFFFFu, M.lo, 0)};
+    int use_tail = 0;
+    if (acc < 0 && sc >= 0) {
+        if (lane == 0 && ff_le(ff_mul(__fmul_rn(w.coin[0], qs), M), w.pc[sc - fc])) acc = sc;
+        acc = __shfl_sync(0xFFFFFFFFu, acc, 0);
+        if (acc < 0) {
+            FF ov{0.0f, 0.0f};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int i = lane + 32 * q;
+                if (i >= TL) continue;
+                const float pt = exp_ff_minus(tx[q], lse);
+                const FF mq = ff_mul(tq[q], M);
+                const FF d = ff_add(FF{pt, 0.0f}, ff_neg(mq));
+                const float dv = __fadd_rn(d.hi, d.lo);
+                const float rh = dv > 0.0f ? dv : 0.0f;
+                w.pt[i] = rh;
+                a.rhat_tail[r * TL + i] = rh;
+                ov = ff_add(ov, (pt < __fadd_rn(mq.hi, mq.lo)) ? FF{pt, 0.0f} : mq);
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) ov = ff_add(ov, ff_shfl_xor(ov, o));
+            M = ff_add(M, ff_neg(ov));
+            use_tail = 1;
+            __syncwarp();
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int i = lane + 32 * q;
+                if (i < nc) w.rc[i] = (cpos[q] >= 0 && cpos[q] < TL) ? w.pt[cpos[q]] : w.pc[i];
+            }
+            __syncwarp();
+        }
+    }
+    if (lane == 0) {
+        const FF M0 = M;
+        if (acc < 0)
+            for (int c2 = 0; c2 < nc; ++c2) {
+                if (w.tok[c2] <= m) continue;  // fills only
+                const float eta = w.coin[1 + w.tok[c2]];
+                const float rv = use_tail ? w.rc[c2] : w.pc[c2];
+                if (ff_le(ff_mul(eta, M), rv)) {
+                    acc = fc + c2;
+                    break;
+                }
+                M = ff_add(M, -rv);
+            }
+        tab[0] = M0.hi;
+        tab[1] = M0.lo;
+        tab[2] = qs;
+        tab[5] = (float)use_tail;
+        tab[6] = (float)acc;
+    }
+}
+
 template <int DT>
 __device__ __noinline__ void finalize_row(const VerifyArgs& a, int64_t r, WarpRow& w) {
     const Dims& n = a.n;
@@ -273,8 +370,9 @@ __device__ __noinline__ void finalize_row(const VerifyArgs& a, int64_t r, WarpRo
         if ((r % NP) == 0 && (!(T > 0.0f) || isinf(T))) atomicOr(a.status, kStBadTemperature);
     }
     // r^ over the tail and the overlap sum of min(p, q~) (sampled child survived)
+    const int variant = a.variant;
     FF ov{0.0f, 0.0f};
-    if (sc >= 0) {
+    if (variant == kVerifyRheo && sc >= 0) {
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             const int i = lane + 32 * q;
@@ -300,7 +398,7 @@ __device__ __noinline__ void finalize_row(const VerifyArgs& a, int64_t r, WarpRo
         const int i = lane + 32 * q;
         if (i >= nc) continue;
         const float p = exp_ff_minus(cx[q], lse);
-        const float rh = (sc >= 0 && cpos[q] >= 0 && cpos[q] < TL) ? w.pt[cpos[q]] : p;
+        const float rh = (variant == kVerifyRheo && sc >= 0 && cpos[q] >= 0 && cpos[q] < TL) ? w.pt[cpos[q]] : p;
         w.pc[i] = p;
         w.rc[i] = rh;
         w.tok[i] = cslot[q];  // the slot decides the coin
@@ -308,6 +406,14 @@ __device__ __noinline__ void finalize_row(const VerifyArgs& a, int64_t r, WarpRo
         tab[kTabP + (K + 1) + i] = rh;
     }
     __syncwarp();
+    if (variant == kVerifyRrsw) {
+        rrsw_walk(a, r, w, nc, fc, sc, qs, cpos, tq, tx, lse, tab);
+        return;
+    }
+    if (variant == kVerifyOneHot) {
+        if (lane == 0) onehot_walk(w, nc, fc, tab);
+        return;
+    }
     if (lane == 0) {
         // Algorithm 1 at this node: stochastic first, then recursive rejection in slot order
         FF M{1.0f, 0.0f};

@@ -16,11 +16,12 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "librheo.so
 
 RHEO_F32, RHEO_BF16 = 0, 1
 RHEO_OK, RHEO_EINVAL, RHEO_ELAUNCH, RHEO_ETOOLARGE = 0, -1, -2, -3
+VERIFY_RHEO, VERIFY_RRSW, VERIFY_ONEHOT = 0, 1, 2
 STATUS_BAD_LOGIT, STATUS_EMPTY_ROW, STATUS_BAD_TEMPERATURE, STATUS_INTERNAL = 1, 2, 4, 8
 SLOT_ROOT, SLOT_LEAD, SLOT_SAMPLED, SLOT_FILL = 0, 1, 2, 3
 
 EXPORTS = ("rheo_sizes", "rheo_workspace_init", "rheo_expand", "rheo_prune", "rheo_verify", "rheo_verify_static",
-           "rheo_tree_attention",
+           "rheo_tree_attention", "rheo_verify_variant",
            "rheo_get_status")
 
 
@@ -82,6 +83,9 @@ def lib():
         L.rheo_verify_static.argtypes = [C, _VP, ctypes.c_int64, _VP, _VP, _VP, ctypes.POINTER(_Tree),
                                          ctypes.POINTER(_Pruned), ctypes.POINTER(_VerifyOut), _VP, _VP]
         L.rheo_get_status.argtypes = [C, _VP, _VP, ctypes.POINTER(ctypes.c_int32)]
+        L.rheo_verify_variant.argtypes = [C, ctypes.c_int32, _VP, ctypes.c_int64, _VP, _VP, _VP,
+                                          ctypes.POINTER(_Tree), ctypes.POINTER(_Pruned), ctypes.POINTER(_VerifyOut),
+                                          _VP, _VP]
         L.rheo_tree_attention.argtypes = [C, ctypes.POINTER(_Pruned), ctypes.POINTER(_TreeAttn), _VP, _VP]
         for name in EXPORTS:
             getattr(L, name).restype = ctypes.c_int
@@ -269,6 +273,18 @@ def verify(cfg: Config, logits: torch.Tensor, temperature: torch.Tensor, seed: t
                              _i64(seed).data_ptr(), _i64(offset).data_ptr(), ctypes.byref(tree.c()),
                              ctypes.byref(pruned.c()), ctypes.byref(out.c()), ws.ptr(), _stream(stream)),
            "rheo_verify")
+
+
+def verify_variant(cfg: Config, variant: int, logits: torch.Tensor, temperature: torch.Tensor, seed: torch.Tensor,
+                   offset: torch.Tensor, tree: Tree, pruned: Pruned, out: VerifyOut, ws: Workspace,
+                   stream=None) -> None:
+    """rheo_verify_variant: VERIFY_RHEO (Algorithm 1), VERIFY_RRSW or VERIFY_ONEHOT."""
+    stride = _rows(cfg, logits, cfg.batch * (cfg.budget + 1))
+    _check(lib().rheo_verify_variant(ctypes.byref(cfg.c()), int(variant), logits.data_ptr(), stride,
+                                     _f32(temperature).data_ptr(), _i64(seed).data_ptr(), _i64(offset).data_ptr(),
+                                     ctypes.byref(tree.c()), ctypes.byref(pruned.c()), ctypes.byref(out.c()),
+                                     ws.ptr(), _stream(stream)),
+           "rheo_verify_variant")
 
 
 def verify_static(cfg: Config, logits: torch.Tensor, temperature: torch.Tensor, seed: torch.Tensor,

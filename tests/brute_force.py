@@ -56,12 +56,16 @@ class Enumerator:
     """Brute force over all sampled-token realisations (Theorem 1, App. C)."""
 
     def __init__(self, V, K, m, S, D, N, T, draft_table, target_table, eps=1e-6,
-                 proxy=None):
+                 proxy=None, verify="rheo"):
         self.V, self.K, self.m, self.S, self.D, self.N, self.T = V, K, m, S, D, N, T
         self.draft = np.asarray(draft_table, dtype=np.float64)
         self.target = np.asarray(target_table, dtype=np.float64)
         self.eps = eps
         self.proxy = proxy  # None: the paper's proxy; a float: a fixed (ad hoc) proxy probability
+        # "rheo": Algorithm 1; "rrsw": recursive rejection, leads first, then the
+        # sampled child, then fills (App. D.2); "onehot": every child a one-hot
+        # candidate in slot order, residual from p (vanilla top-K, App. A)
+        self.verify = verify
 
     # -- one pool (Sec. 3.2, App. C.1) ------------------------------------
     def support(self, row):
@@ -177,25 +181,46 @@ class Enumerator:
             return
         s = next((n for n in kids if n.kind == "sampled"), None)
         reach = weight
+        if self.verify == "onehot":
+            s = None
+        qt = np.zeros(self.V)
         if s is not None:
-            a = min(1.0, p[s.token] / s.qtilde)
-            self.walk(nodes, keep, s.gen, prefix + (s.token,), L, reach * a, out, acc, depth + 1)
-            reach *= 1.0 - a
-            qt = np.zeros(self.V)
             for v, q in nodes[g].tail.items():
                 qt[v] = q
-            rhat = np.maximum(0.0, p - qt)
-        else:
-            rhat = p.copy()
+        rhat = p.copy()
         M = rhat.sum()
-        for c in kids:
-            if c is s:
-                continue
+
+        def one_hot(c):  # accept c with probability r^(c) / M, else drop it from r^
+            nonlocal reach, M
             a = rhat[c.token] / M if M > 0 else 1.0
             self.walk(nodes, keep, c.gen, prefix + (c.token,), L, reach * a, out, acc, depth + 1)
             reach *= 1.0 - a
             M -= rhat[c.token]
             rhat[c.token] = 0.0
+
+        if self.verify == "rrsw":
+            for c in kids:
+                if c.kind == "lead":
+                    one_hot(c)
+            if s is not None:
+                a = min(1.0, (rhat[s.token] / M) / s.qtilde) if M > 0 else 1.0
+                self.walk(nodes, keep, s.gen, prefix + (s.token,), L, reach * a, out, acc, depth + 1)
+                reach *= 1.0 - a
+                rhat = np.maximum(0.0, rhat - M * qt)
+                M = rhat.sum()
+            for c in kids:
+                if c.kind == "fill":
+                    one_hot(c)
+        else:
+            if s is not None:
+                a = min(1.0, p[s.token] / s.qtilde)
+                self.walk(nodes, keep, s.gen, prefix + (s.token,), L, reach * a, out, acc, depth + 1)
+                reach *= 1.0 - a
+                rhat = np.maximum(0.0, p - qt)
+                M = rhat.sum()
+            for c in kids:
+                if c is not s:
+                    one_hot(c)
         acc[depth] += reach
         for c in kids:
             rhat[c.token] = 0.0

@@ -56,7 +56,7 @@ class Side:
 
 
 def run_gpu(w: synth.Workload, draft: synth.DraftInputs, cfg: rheo.Config, target_override=None,
-            row_stride_pad: int = 0) -> Side:
+            row_stride_pad: int = 0, variant: int = 0) -> Side:
     tree = rheo.Tree(cfg)
     pr = rheo.Pruned(cfg)
     out = rheo.VerifyOut(cfg)
@@ -79,7 +79,10 @@ def run_gpu(w: synth.Workload, draft: synth.DraftInputs, cfg: rheo.Config, targe
         padded = torch.zeros((B, NP, V + row_stride_pad), dtype=tgt.dtype, device=tgt.device)
         padded[..., :V] = tgt
         tgt = padded[..., :V]
-    rheo.verify(cfg, tgt, draft.temperature, draft.seed, draft.offset, tree, pr, out, ws)
+    if variant:
+        rheo.verify_variant(cfg, variant, tgt, draft.temperature, draft.seed, draft.offset, tree, pr, out, ws)
+    else:
+        rheo.verify(cfg, tgt, draft.temperature, draft.seed, draft.offset, tree, pr, out, ws)
     st = rheo.status(cfg, ws)
     c = lambda t: t.cpu().numpy()
     return Side(c(tree.token), c(tree.parent), c(tree.slot), c(tree.score), c(tree.log_proxy), c(tree.qtilde),
@@ -90,11 +93,12 @@ def run_gpu(w: synth.Workload, draft: synth.DraftInputs, cfg: rheo.Config, targe
                 c(out.row_lse), st)
 
 
-def run_oracle(w: synth.Workload, draft: synth.DraftInputs, cfg: rheo.Config, reqs, target_override=None) -> Side:
+def run_oracle(w: synth.Workload, draft: synth.DraftInputs, cfg: rheo.Config, reqs, target_override=None,
+               variant: int = 0) -> Side:
     """The oracle on requests `reqs` (a sub-batch of the same inputs)."""
     reqs = list(reqs)
     ocfg = oracle.Config(B=len(reqs), V=cfg.vocab, K=cfg.K, m=cfg.m, S=cfg.support, D=cfg.depth, N=cfg.budget,
-                         eps=cfg.eps)
+                         eps=cfg.eps, verify_mode=variant)
     T = draft.temperature.cpu().numpy()[reqs]
     seed = u64(draft.seed)[reqs]
     off = u64(draft.offset)[reqs]

@@ -445,6 +445,28 @@ def main(argv=None):
         variants[name]["mean_accepted"] = sum(acc) / len(acc)
         variants[name]["samples"] = len(acc)
 
+    # synthetic analogue of the ablations over m and T (Sec. 5.3, Sec. 5.4):
+    # multi-cycle decoding against k-gram draft / target models (V = 64, k = 2),
+    # tau = mean tokens emitted per cycle
+    from paper_2609_21827_gb300 import cycles as cyc
+    lm_gen = torch.Generator().manual_seed(2609)
+    d_lm = cyc.KGramLM.random(64, 2, 1.5, lm_gen, device=device)
+    t_lm = cyc.KGramLM.random(64, 2, 1.5, lm_gen, device=device, base=d_lm, noise=0.8)
+    tau = {}
+    lm_ms = 0.0
+    for m_ in (0, 1, 2, 3):
+        for T_ in (0.5, 1.0):
+            c2 = rheo.Config(batch=1024, vocab=64, K=8, depth=6, budget=40, m=m_, support=64, dtype="f32")
+            win = torch.randint(0, 64, (1024, 2), generator=lm_gen).to(device)
+            sd = torch.arange(1024, dtype=torch.int64, device=device) * 7919 + 31 * m_ + int(10 * T_)
+            t0 = time.time()
+            res = cyc.run_cycles(c2, d_lm, t_lm, win, torch.full((1024,), T_), sd, cycles=6, L=1)
+            torch.cuda.synchronize()
+            lm_ms += (time.time() - t0) * 1e3 / 6
+            tau[f"m{m_}_T{T_}"] = float(res.accepted.float().mean().item()) + 1.0
+    synthetic_lm = {"vocab": 64, "k": 2, "K": 8, "depth": 6, "budget": 40, "sequences": 1024, "cycles": 6,
+                    "tau": tau, "host_ms_per_cycle": lm_ms / 8}
+
     # end to end through the public API with host buffers: H2D of every input, D2H of the results
     e2e = None
     if rank == 0 or world > 1:
@@ -528,6 +550,7 @@ def main(argv=None):
                     "step_frac_of_peak": step_gbs / peak,
                     "tree_attention_us": attn_us,
                     "verify_variants": variants,
+                    "synthetic_lm": synthetic_lm,
                     "tree_attention_bytes": w.batch * (w.budget + 1) * ((w.budget + 1) + 4 + 4 * (w.depth + 1) + 12)},
         "clocks": clocks,
         "gpu_launches": args.steps * (D + 4),  # D expand, 1 prune, 3 verify (prep, stream, residual)

@@ -1,0 +1,105 @@
+"""Multi-cycle decoding on the GPU path against synthetic k-gram models.
+
+Theorem 1 says the emitted tokens follow the target model whatever the draft:
+the first two emitted tokens of many independent sequences are compared with
+the target's exact law (chi-square).  Theorem 2 (App. D.1) gives the
+acceptance probability of a single layer with nothing pruned in closed form: at
+D = 1 the mean acceptance over all visited contexts is compared with the
+average of that formula over the same contexts.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+from scipy import stats
+
+from paper_2609_21827_gb300 import build, cycles, rheo
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    build.build()
+
+
+def _models(V, k, seed, noise=0.8):
+    g = torch.Generator().manual_seed(seed)
+    draft = cycles.KGramLM.random(V, k, 1.5, g)
+    target = cycles.KGramLM.random(V, k, 1.5, g, base=draft, noise=noise)
+    return draft, target
+
+
+def _chisq_p(obs, exp):
+    keep = exp >= 5
+    o = np.append(obs[keep], obs[~keep].sum())
+    e = np.append(exp[keep], exp[~keep].sum())
+    if e[-1] == 0:
+        o, e = o[:-1], e[:-1]
+    return stats.chisquare(o, e * o.sum() / e.sum()).pvalue
+
+
+@pytest.mark.parametrize("variant", [rheo.VERIFY_RHEO, rheo.VERIFY_RRSW, rheo.VERIFY_ONEHOT])
+@pytest.mark.parametrize("m,T", [(1, 1.0), (0, 0.7), (2, 1.3)])
+def test_first_two_tokens_follow_the_target(variant, m, T):
+    V, k, B = 16, 1, 6000
+    draft, target = _models(V, k, seed=100 + m)
+    cfg = rheo.Config(batch=B, vocab=V, K=3, depth=3, budget=8, m=m, support=V, dtype="f32")
+    counts = np.zeros(V * V)
+    for rep in range(2):
+        window = torch.full((B, k), 3, dtype=torch.int64, device="cuda")
+        seed = torch.arange(B, dtype=torch.int64, device="cuda") * 7919 + 1000003 * rep + 17
+        res = cycles.run_cycles(cfg, draft, target, window, torch.full((B,), T), seed, cycles=2, L=2,
+                                variant=variant)
+        st = res.streams.cpu().numpy()
+        assert (st >= 0).all()
+        counts += np.bincount(st[:, 0] * V + st[:, 1], minlength=V * V)
+    tab = target.table.cpu().double().numpy() / T
+    p1 = np.exp(tab[3] - tab[3].max()); p1 /= p1.sum()
+    law = np.zeros(V * V)
+    for a in range(V):
+        p2 = np.exp(tab[a] - tab[a].max()); p2 /= p2.sum()
+        law[a * V:(a + 1) * V] = p1[a] * p2
+    assert _chisq_p(counts, law * counts.sum()) > 0.01
+
+
+def _thm2(p, order, qt, n):
+    """App. D.1: acceptance of one layer of n = K+1 slots with nothing pruned."""
+    top = order[: n - 1]
+    rest = [v for v in range(len(p)) if v not in top]
+    r = np.maximum(0.0, p - qt)
+    r = r / r.sum()
+    return (sum(p[v] for v in top) + sum(min(p[v], qt[v]) for v in rest)
+            + r[order[n - 1]] * sum(max(0.0, qt[v] - p[v]) for v in top))
+
+
+@pytest.mark.parametrize("K,m,T", [(2, 1, 1.0), (3, 1, 0.7), (3, 0, 1.0)])
+def test_single_layer_acceptance_matches_theorem2_across_cycles(K, m, T):
+    V, k, B, C = 24, 1, 4000, 6
+    draft, target = _models(V, k, seed=200 + K + m, noise=1.0)
+    cfg = rheo.Config(batch=B, vocab=V, K=K, depth=1, budget=K + 1, m=m, support=V, dtype="f32")
+    window = torch.randint(0, V, (B, k), generator=torch.Generator().manual_seed(5)).cuda()
+    seed = torch.arange(B, dtype=torch.int64, device="cuda") * 104729 + 11
+    res = cycles.run_cycles(cfg, draft, target, window, torch.full((B,), T), seed, cycles=C, L=1)
+    acc = res.accepted.cpu().numpy().astype(np.float64)
+    wins = res.windows.cpu().numpy()[:, :, -1]
+    dtab = draft.table.cpu().double().numpy()
+    ttab = target.table.cpu().double().numpy()
+    expect = np.zeros(V)
+    for ctx in range(V):
+        row = dtab[ctx]
+        order = sorted(range(V), key=lambda v: (-row[v], v))
+        qt = np.zeros(V)
+        t = row[order[m:]] / T
+        e = np.exp(t - t.max())
+        qt[order[m:]] = e / e.sum()
+        pt = np.exp(ttab[ctx] / T - (ttab[ctx] / T).max())
+        pt /= pt.sum()
+        expect[ctx] = _thm2(pt, order, qt, K + 1)
+    want = expect[wins].mean()
+    got = acc.mean()
+    sd = math.sqrt(max(want * (1 - want), 1e-12) / acc.size)
+    assert abs(got - want) <= 5 * sd, (got, want, sd)

@@ -61,7 +61,7 @@ _P = ctypes.c_void_p
 class _Tree(ctypes.Structure):
     _fields_ = [(n, _P) for n in (
         "token", "parent", "log_proxy", "score", "qtilde", "slot", "frontier",
-        "tail_ids", "tail_q", "lse1", "gap_sample", "gap_frontier")]
+        "tail_ids", "tail_q", "lse1", "gap_sample", "gap_frontier", "lse_tail")]
 
 
 class _Pruned(ctypes.Structure):
@@ -146,7 +146,7 @@ class Config:
 
     @property
     def TL(self) -> int:
-        return self.S - self.m
+        return (self.V if self.S == 0 else self.S) - self.m
 
     def rows_at(self, d: int) -> int:
         return 1 if d == 1 else self.K
@@ -170,6 +170,7 @@ class Tree:
     lse1: np.ndarray = field(init=False)
     gap_sample: np.ndarray = field(init=False)
     gap_frontier: np.ndarray = field(init=False)
+    lse_tail: np.ndarray = field(init=False)
 
     def __post_init__(self):
         c = self.cfg
@@ -186,6 +187,7 @@ class Tree:
         self.lse1 = np.zeros((B, E), np.float32)
         self.gap_sample = np.full((B, E), np.inf)
         self.gap_frontier = np.full((B, c.D), np.inf)
+        self.lse_tail = np.zeros((B, E), np.float32)
 
     def c(self) -> _Tree:
         return _Tree(*[_ptr(getattr(self, n)) for n, _ in _Tree._fields_])

@@ -52,7 +52,8 @@ int64_t orc_expansions_per_request(const orc_cfg* c) { return 1 + (int64_t)(c->D
 int orc_check_cfg(const orc_cfg* c) {
     if (!c) return -1;
     if (c->B < 1 || c->V < 1 || c->K < 0 || c->m < 0 || c->m > c->K) return -1;
-    if (c->S < c->K + 1 || c->S > c->V || c->S > 128) return -1;
+    if (c->S != 0 && (c->S < c->K + 1 || c->S > c->V || c->S > 128)) return -1;
+    if (c->S == 0 && c->V < c->K + 1) return -1;
     if (c->D < 1 || (c->K == 0 && c->D > 1)) return -1;
     int64_t G1 = orc_nodes_per_request(c);
     if (G1 > ORC_MAX_NODES) return -1;
@@ -61,6 +62,11 @@ int orc_check_cfg(const orc_cfg* c) {
     if (c->verify_mode < ORC_VERIFY_RHEO || c->verify_mode > ORC_VERIFY_ONEHOT) return -1;
     return 0;
 }
+
+/* Support size: S, or the whole vocabulary when S == 0 ("full support",
+ * App. B Table tab:sparse_support, row Full).  In full support the tail draw
+ * of token v uses draw index v (the token id) instead of its tail position. */
+static int support_of(const orc_cfg* c) { return c->S == 0 ? c->V : c->S; }
 
 static int64_t depth_base(const orc_cfg* c, int d) {
     return d == 1 ? 1 : 1 + (int64_t)(c->K + 1) + (int64_t)(d - 2) * c->K * (c->K + 1);
@@ -171,7 +177,7 @@ int orc_topk_row(const float* row, int32_t V, int32_t S, int32_t* ids_out) {
  * (NaN / +inf entry, or fewer than m+1 finite logits). */
 static int expand_row(const orc_cfg* c, int d, int b, int f, const float* l, float T, uint64_t seed,
                       uint64_t offset, orc_tree* t) {
-    const int K = c->K, m = c->m, S = c->S, V = c->V, TL = S - m;
+    const int K = c->K, m = c->m, S = support_of(c), V = c->V, TL = S - m;
     const int64_t G1 = orc_nodes_per_request(c), E = orc_expansions_per_request(c);
     const int64_t par = (d == 1) ? 0 : t->frontier[(int64_t)b * K + f];
     const int64_t e = (d == 1) ? 0 : 1 + (int64_t)(d - 2) * K + f;
@@ -200,12 +206,14 @@ static int expand_row(const orc_cfg* c, int d, int b, int f, const float* l, flo
     for (int v = 0; v < V; ++v) { srt[v].l = l[v]; srt[v].id = v; }
     qsort(srt, (size_t)V, sizeof(orc_entry), cmp_entry);
 
-    float lq0[128];
+    float* lq0 = (float*)malloc(sizeof(float) * (size_t)S * 3);
+    if (!lq0) { free(srt); return -2; }
+    float* tau = lq0 + S;
+    float* qt = tau + S;
     for (int i = 0; i < S; ++i) lq0[i] = srt[i].l - lse1; /* fp32 */
 
     /* tempered tail q~ over support ranks m+1..S (App. C.1: q~ = q / z on the
      * complement of the leads; Sec. 5.4: temperature applies to sampling) */
-    float tau[128];
     double mt = -INFINITY;
     for (int i = 0; i < TL; ++i) {
         tau[i] = srt[m + i].l / T; /* fp32 division */
@@ -214,19 +222,24 @@ static int expand_row(const orc_cfg* c, int d, int b, int f, const float* l, flo
     double st = 0.0;
     for (int i = 0; i < TL; ++i) st += exp((double)tau[i] - mt);
     const double lse_tail = mt + log(st);
-    float qt[128];
     for (int i = 0; i < TL; ++i) qt[i] = (float)exp((double)tau[i] - lse_tail);
+    if (t->lse_tail) t->lse_tail[(int64_t)b * E + e] = (float)lse_tail;
 
-    /* Y ~ q~ by Gumbel-max; ties keep the earlier tail position */
+    /* Y ~ q~ by Gumbel-max; ties keep the earlier tail position (full support:
+     * the lower token id) */
     int best = -1;
     float bk = -INFINITY, second = -INFINITY;
     for (int i = 0; i < TL; ++i) {
-        float g = gumbel(orc_uniform(seed, offset, ORC_TAG_SAMPLE, (int32_t)par, (uint64_t)i));
+        const uint64_t draw = (c->S == 0) ? (uint64_t)srt[m + i].id : (uint64_t)i;
+        float g = gumbel(orc_uniform(seed, offset, ORC_TAG_SAMPLE, (int32_t)par, draw));
         float key = tau[i] + g;
-        if (key > bk) { second = bk; bk = key; best = i; }
-        else if (key > second) second = key;
+        if (key > bk || (c->S == 0 && key == bk && best >= 0 && srt[m + i].id < srt[m + best].id)) {
+            second = bk;
+            bk = key;
+            best = i;
+        } else if (key > second) second = key;
     }
-    if (best < 0) { free(srt); return -2; }
+    if (best < 0) { free(srt); free(lq0); return -2; }
 
     /* construction probability of Y (Sec. 3.2; App. C.1):
      *   m >= 1: min{q(x_m), z}, z = 1 - sum_{i<=m} q(x_i); never below
@@ -293,6 +306,7 @@ static int expand_row(const orc_cfg* c, int d, int b, int f, const float* l, flo
     t->lse1[(int64_t)b * E + e] = lse1;
     t->gap_sample[(int64_t)b * E + e] = rel_gap(bk, second);
     free(srt);
+    free(lq0);
     return 0;
 }
 
@@ -479,7 +493,7 @@ static int verify_variant(const orc_cfg* c, int b, const float* l, double lu, fl
                           uint64_t offset, const orc_tree* t, const orc_pruned* p, int u, double* gap_out,
                           float* rhat, int32_t* tail_pos, const int32_t** tids_out, double* M_out,
                           int* use_tail_out) {
-    const int N = c->N, TL = c->S - c->m;
+    const int N = c->N, TL = support_of(c) - c->m;
     const int64_t G1 = orc_nodes_per_request(c), E = orc_expansions_per_request(c);
     const int64_t nb = (int64_t)b * G1, pb = (int64_t)b * (N + 1);
     const int fc = p->first_child[pb + u], nc = p->n_child[pb + u], sc = p->sampled_child[pb + u];
@@ -552,7 +566,7 @@ done:
 
 static int verify_request(const orc_cfg* c, int b, const float* target, float T, uint64_t seed,
                           uint64_t offset, const orc_tree* t, const orc_pruned* p, orc_verify_out* o) {
-    const int V = c->V, N = c->N, D = c->D, K = c->K, TL = c->S - c->m;
+    const int V = c->V, N = c->N, D = c->D, K = c->K, TL = support_of(c) - c->m;
     const int64_t G1 = orc_nodes_per_request(c), E = orc_expansions_per_request(c);
     const int64_t nb = (int64_t)b * G1, pb = (int64_t)b * (N + 1);
     const float* rows = target + pb * V;
@@ -739,7 +753,7 @@ int orc_run_prefix_lm(const orc_cfg* c0, const float* draft_table, const float* 
     orc_cfg c = *c0;
     c.B = 1;
     if (orc_check_cfg(&c) || table_depth < c.D || table_depth < L - 1 || L < 1) return -1;
-    const int V = c.V, K = c.K, D = c.D, N = c.N, TL = c.S - c.m;
+    const int V = c.V, K = c.K, D = c.D, N = c.N, TL = support_of(&c) - c.m;
     const int64_t G1 = orc_nodes_per_request(&c), E = orc_expansions_per_request(&c);
     int err = 0;
 #pragma omp parallel for schedule(static) reduction(| : err)
@@ -760,6 +774,7 @@ int orc_run_prefix_lm(const orc_cfg* c0, const float* draft_table, const float* 
         t.lse1 = (float*)malloc(sizeof(float) * E);
         t.gap_sample = (double*)malloc(sizeof(double) * E);
         t.gap_frontier = (double*)malloc(sizeof(double) * D);
+        t.lse_tail = NULL;
         int32_t* pbuf = (int32_t*)malloc(sizeof(int32_t) * 7 * (N + 1));
         p.gen_id = pbuf; p.token = pbuf + (N + 1); p.parent = pbuf + 2 * (N + 1);
         p.depth = pbuf + 3 * (N + 1); p.first_child = pbuf + 4 * (N + 1);

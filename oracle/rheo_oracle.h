@@ -39,7 +39,8 @@ typedef struct {
     int32_t V;       /* vocabulary */
     int32_t K;       /* deterministic slots per pool; pool size K+1 */
     int32_t m;       /* lead tokens (the rheostat), 0 <= m <= K */
-    int32_t S;       /* sparse support, K+1 <= S <= min(V,128) */
+    int32_t S;       /* sparse support, K+1 <= S <= min(V,128); 0: the whole vocabulary
+                        (full support: tail draws indexed by token id) */
     int32_t D;       /* expansion depth */
     int32_t N;       /* prune budget (non-root nodes kept) */
     double eps;      /* proxy offset for m = 0 */
@@ -72,6 +73,7 @@ typedef struct {
     float* lse1;         /* [B*E] log-partition of the untempered draft row */
     double* gap_sample;  /* [B*E] relative gap of the two best Gumbel keys */
     double* gap_frontier;/* [B*D] relative gap at the frontier boundary of depth d (index d-1) */
+    float* lse_tail;     /* [B*E] log sum over the tail of exp(l/T), or NULL */
 } orc_tree;
 
 typedef struct {

@@ -1,0 +1,79 @@
+"""Pins of the oracle's full-support mode (S = V; App. B, Table tab:sparse_support,
+row Full): the sampled token is drawn from the tempered draft distribution over
+the whole vocabulary minus the leads, with draw index = token id.
+
+Pinned against scipy's softmax, the law of Y (chi-square over seeds), and the
+exhaustive enumeration of brute_force.py, whose law of trees with S = V does
+not depend on how the uniforms are indexed: the acceptance and the emitted
+two-token law of the oracle's Monte-Carlo runs must match it.
+"""
+import math
+
+import numpy as np
+import pytest
+from scipy import special, stats
+
+import brute_force as bf
+import oracle
+
+
+def _chisq_p(obs, exp):
+    keep = exp >= 5
+    o = np.append(obs[keep], obs[~keep].sum())
+    e = np.append(exp[keep], exp[~keep].sum())
+    if e[-1] == 0:
+        o, e = o[:-1], e[:-1]
+    return stats.chisquare(o, e * o.sum() / e.sum()).pvalue
+
+
+def test_tail_distribution_and_lse_against_scipy():
+    rng = np.random.default_rng(3)
+    V, K, m, B, T = 300, 4, 2, 3, 0.8
+    cfg = oracle.Config(B=B, V=V, K=K, m=m, S=0, D=1, N=K + 1)
+    tree = oracle.Tree(cfg)
+    rows = (rng.normal(size=(B, 1, V)) * 2).astype(np.float32)
+    oracle.expand(cfg, 1, rows, np.full(B, T, np.float32), rng.integers(1, 2**62, size=B, dtype=np.uint64),
+                  np.zeros(B, np.uint64), tree)
+    for b in range(B):
+        l = rows[b, 0].astype(np.float64)
+        order = np.lexsort((np.arange(V), -rows[b, 0]))
+        tail = order[m:]
+        np.testing.assert_array_equal(tree.tail_ids[b, 0], tail)
+        tau = (rows[b, 0][tail] / np.float32(T)).astype(np.float64)
+        np.testing.assert_allclose(tree.tail_q[b, 0], special.softmax(tau), rtol=2e-6, atol=1e-12)
+        assert abs(tree.lse_tail[b, 0] - special.logsumexp(tau)) < 2e-6
+        assert abs(tree.lse1[b, 0] - special.logsumexp(l)) < 2e-6
+
+
+def test_sampled_token_law():
+    V, K, m, T, n = 16, 2, 1, 0.9, 40000
+    rng = np.random.default_rng(9)
+    row = (rng.normal(size=V) * 1.5).astype(np.float32)
+    cfg = oracle.Config(B=n, V=V, K=K, m=m, S=0, D=1, N=K + 1)
+    tree = oracle.Tree(cfg)
+    rows = np.broadcast_to(row, (n, 1, V)).copy()
+    seeds = np.arange(1, n + 1, dtype=np.uint64) * np.uint64(2654435761)
+    oracle.expand(cfg, 1, rows, np.full(n, T, np.float32), seeds, np.zeros(n, np.uint64), tree)
+    ys = tree.token[:, 1 + m]  # slot m of the root's children (gen ids 1..K+1)
+    order = np.lexsort((np.arange(V), -row))
+    q = np.zeros(V)
+    q[order[m:]] = special.softmax((row[order[m:]] / np.float32(T)).astype(np.float64))
+    assert _chisq_p(np.bincount(ys, minlength=V), q * n) > 0.01
+
+
+@pytest.mark.parametrize("K,m,T,D,N", [(2, 1, 1.0, 1, 3), (3, 0, 0.7, 2, 6), (2, 2, 1.2, 2, 5)])
+def test_monte_carlo_against_enumeration(K, m, T, D, N):
+    V, n = 12, 200000
+    rng = np.random.default_rng(40 + K + m)
+    dr, tg = bf.random_tables(rng, V, D)
+    cfg = oracle.Config(B=1, V=V, K=K, m=m, S=0, D=D, N=N)
+    st, acc = oracle.run_prefix_lm(cfg, dr, tg, D, n, T, 31337, 2)
+    en = bf.Enumerator(V, K, m, V, D, N, T, dr, tg)
+    _, accl = en.stream_distribution(2)
+    ea = np.array([accl.get(i, 0.0) for i in range(D + 1)])
+    assert _chisq_p(np.bincount(acc, minlength=D + 1), ea * n) > 0.01
+    tl = en.target_law(2)
+    p2 = np.zeros(V * V)
+    for (a, b), pr in tl.items():
+        p2[a * V + b] += pr
+    assert _chisq_p(np.bincount(st[:, 0] * V + st[:, 1], minlength=V * V), p2 * n) > 0.01

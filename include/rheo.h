@@ -60,7 +60,13 @@ enum {
 
 /* Problem size.  K = deterministic slots per pool (pool = K+1), 0 <= m <= K,
  * K+1 <= support <= min(vocab, 128), depth >= 1 (depth 1 if K = 0),
- * 1 <= budget <= G1-1, G1 <= 16384, vocab <= 262144, eps > 0 when m = 0. */
+ * 1 <= budget <= G1-1, G1 <= 16384, vocab <= 262144, eps > 0 when m = 0.
+ * support = 0 selects full support (App. B, Table tab:sparse_support, row
+ * Full): the sampled token is drawn from the tempered draft distribution over
+ * the whole vocabulary minus the leads, with Philox draw index = token id
+ * (sparse support: its tail position); requires m <= 1 and K+1 <= 128; no tail
+ * lists are kept (tail_ids / tail_q unused, lse_tail required) and the tree is
+ * verified by rheo_verify_full, which re-reads the expanded nodes' draft rows. */
 typedef struct {
     int32_t batch;   /* B requests                                  */
     int32_t vocab;   /* V                                           */
@@ -87,6 +93,9 @@ typedef struct {
     int32_t* tail_ids;  /* [B,E,S-m] support ranks m+1..S of each expanded node        */
     float* tail_q;      /* [B,E,S-m] q~ over that tail: softmax(l/T) renormalised      */
     float* lse1;        /* [B,E] log sum_v exp(l_v) of each expanded draft row         */
+    float* lse_tail;    /* [B,E] log of the tail's sum of exp(l/T) (ranks m+1..S, or V
+                           minus the leads with full support); may be NULL with sparse
+                           support, required with full support                          */
 } rheo_tree;
 
 /* Pruned tree, written by rheo_prune: [B, N+1], root first, ascending gen id. */

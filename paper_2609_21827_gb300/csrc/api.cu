@@ -30,7 +30,11 @@ bool valid(const rheo_config* c) {
     if (c->dtype != RHEO_F32 && c->dtype != RHEO_BF16) return false;
     if (c->batch < 1 || c->vocab < 1 || c->vocab > kMaxVocab) return false;
     if (c->K < 0 || c->m < 0 || c->m > c->K) return false;
-    if (c->support < c->K + 1 || c->support > c->vocab || c->support > kMaxSupport) return false;
+    if (c->support == 0) {  // full support: the sampled token over the whole vocabulary
+        if (c->K + 1 > c->vocab || c->K + 1 > kMaxSupport || c->m > 1) return false;
+    } else if (c->support < c->K + 1 || c->support > c->vocab || c->support > kMaxSupport) {
+        return false;
+    }
     if (c->depth < 1 || (c->K == 0 && c->depth > 1)) return false;
     const int64_t G1 = nodes_per_request(*c);
     if (G1 > kMaxNodes) return false;
@@ -51,8 +55,8 @@ struct Layout {
 size_t up(size_t x) { return (x + 255) & ~(size_t)255; }
 
 Layout layout(const rheo_config& c) {
-    const int64_t B = c.batch, F = c.K > 0 ? c.K : 1, P = tiles_per_row(c), S = c.support;
-    const int64_t NP = c.budget + 1, TL = c.support - c.m;
+    const int64_t B = c.batch, F = c.K > 0 ? c.K : 1, P = tiles_per_row(c), S = c.support == 0 ? c.K + 1 : c.support;
+    const int64_t NP = c.budget + 1, TL = c.support == 0 ? 0 : c.support - c.m;
     const int64_t VC = verify_chunks_per_row(c.dtype == RHEO_BF16 ? 1 : 0, c.vocab);
     Layout L{};
     size_t o = 0;
@@ -110,7 +114,9 @@ bool rows_aligned(const void* p, int64_t row_stride, const rheo_config& c) {
 Dims dims(const rheo_config& c) {
     Dims n;
     n.B = c.batch; n.V = c.vocab; n.K = c.K; n.m = c.m; n.S = c.support; n.D = c.depth; n.N = c.budget;
-    n.TL = c.support - c.m;
+    n.full = c.support == 0 ? 1 : 0;
+    if (n.full) n.S = c.K + 1;  // ranks selected: the leads and the fill candidates
+    n.TL = n.full ? 0 : c.support - c.m;
     n.GW = (c.K + 1) + n.TL;
     n.chunks = tiles_per_row(c);
     n.G1 = nodes_per_request(c);
@@ -119,9 +125,10 @@ Dims dims(const rheo_config& c) {
     return n;
 }
 
-bool tree_ok(const rheo_tree* t) {
-    return t && t->token && t->parent && t->log_proxy && t->score && t->qtilde && t->slot && t->frontier &&
-           t->tail_ids && t->tail_q && t->lse1;
+bool tree_ok(const rheo_tree* t, const rheo_config& c) {
+    if (!(t && t->token && t->parent && t->log_proxy && t->score && t->qtilde && t->slot && t->frontier && t->lse1))
+        return false;
+    return c.support == 0 ? t->lse_tail != nullptr : (t->tail_ids && t->tail_q);
 }
 bool pruned_ok(const rheo_pruned* p) {
     return p && p->gen_id && p->token && p->parent && p->depth && p->first_child && p->n_child && p->sampled_child;
@@ -129,7 +136,7 @@ bool pruned_ok(const rheo_pruned* p) {
 
 TreePtrs tree_ptrs(const rheo_tree* t) {
     return TreePtrs{t->token, t->parent, t->log_proxy, t->score, t->qtilde, t->slot,
-                    t->frontier, t->tail_ids, t->tail_q, t->lse1};
+                    t->frontier, t->tail_ids, t->tail_q, t->lse1, t->lse_tail};
 }
 PrunedPtrs pruned_ptrs(const rheo_pruned* p) {
     return PrunedPtrs{p->gen_id, p->token, p->parent, p->depth, p->first_child, p->n_child, p->sampled_child};
@@ -159,7 +166,7 @@ extern "C" int rheo_expand(const rheo_config* cfg, int32_t d, const void* logits
                            const float* temperature, const uint64_t* seed, const uint64_t* offset,
                            const rheo_tree* tree, void* ws, rheo_stream_t stream) {
     if (!valid(cfg) || d < 1 || d > cfg->depth || !logits || row_stride < cfg->vocab || !temperature || !seed ||
-        !offset || !tree_ok(tree) || !ws)
+        !offset || !tree_ok(tree, *cfg) || !ws)
         return RHEO_EINVAL;
     const Layout L = layout(*cfg);
     ExpandArgs a;
@@ -186,17 +193,20 @@ extern "C" int rheo_expand(const rheo_config* cfg, int32_t d, const void* logits
     // one segment and P = 1 needs no merge.  More rows: one CTA per SM, rows
     // cut where the even split of the tiles falls.
     int grid;
-    if (rows <= sms) {
+    if (cfg->support == 0) {
+        grid = (int)rows;  // full support: one CTA per row, no merge of partial Gumbel keys
+    } else if (rows <= sms) {
         const int64_t P = std::max<int64_t>(1, std::min<int64_t>(tpr, sms / rows));
         grid = (int)(rows * P);
     } else {
         grid = (int)std::min<int64_t>(rows * tpr, (int64_t)sms);
     }
     const int segs = max_segments(rows, tpr, grid);
-    a.keys_bytes = expand_keys_bytes(segs, cfg->support);
-    const size_t smem = expand_smem_bytes(segs, cfg->support);
+    a.keys_bytes = expand_keys_bytes(segs, a.n.S);
+    const size_t smem = expand_smem_bytes(segs, a.n.S);
     if (smem + 8 * 1024 > 227 * 1024) return RHEO_EINVAL;
-    return launch_expand(a, cfg->dtype, rows_aligned(logits, row_stride, *cfg), grid, smem, (cudaStream_t)stream) ==
+    return launch_expand(a, cfg->dtype, rows_aligned(logits, row_stride, *cfg), cfg->support == 0, grid, smem,
+                         (cudaStream_t)stream) ==
                    cudaSuccess
                ? RHEO_OK
                : RHEO_ELAUNCH;
@@ -204,7 +214,7 @@ extern "C" int rheo_expand(const rheo_config* cfg, int32_t d, const void* logits
 
 extern "C" int rheo_prune(const rheo_config* cfg, const rheo_tree* tree, const rheo_pruned* pruned, void* ws,
                           rheo_stream_t stream) {
-    if (!valid(cfg) || !tree_ok(tree) || !pruned_ok(pruned) || !ws) return RHEO_EINVAL;
+    if (!valid(cfg) || !tree_ok(tree, *cfg) || !pruned_ok(pruned) || !ws) return RHEO_EINVAL;
     const Layout L = layout(*cfg);
     PruneArgs a;
     a.n = dims(*cfg);
@@ -241,7 +251,8 @@ extern "C" int rheo_verify_variant(const rheo_config* cfg, int32_t variant, cons
                                    const rheo_tree* tree, const rheo_pruned* pruned, const rheo_verify_out* out,
                                    void* ws, rheo_stream_t stream) {
     if (variant != RHEO_VERIFY_RHEO && variant != RHEO_VERIFY_RRSW && variant != RHEO_VERIFY_ONEHOT) return RHEO_EINVAL;
-    if (!valid(cfg) || !logits || row_stride < cfg->vocab || !temperature || !seed || !offset || !tree_ok(tree) ||
+    if (cfg && cfg->support == 0) return RHEO_EINVAL;  // full support verifies through rheo_verify_full
+    if (!valid(cfg) || !logits || row_stride < cfg->vocab || !temperature || !seed || !offset || !tree_ok(tree, *cfg) ||
         !pruned_ok(pruned) || !out || !out->accepted_len || !out->accepted_tokens || !out->accepted_nodes ||
         !out->bonus_token || !ws)
         return RHEO_EINVAL;

@@ -52,9 +52,13 @@ struct E2Smem {
     float lq0[kMaxSupport];
     float q[kMaxSupport];
     float lp;
-    int best;
+    int best;    // sparse support: tail position of Y; full support: its support rank, or -1
     float lse1;
     int bad;
+    float lse_tail;
+    int yid;     // full support: the sampled token
+    float qy;    // full support: q~(Y)
+    unsigned long long gk[4];  // full support: the best Gumbel keys of the row
 };
 
 struct HistSel {
@@ -441,7 +445,11 @@ __device__ __forceinline__ void stage_flush(unsigned long long* region, int& cnt
 
 }  // namespace
 
-template <int DT, bool ALIGNED>
+// Gumbel keys each thread keeps in full support: the m+1 best (m <= 1), so
+// that one of them is not the lead
+constexpr int kGumbelKeep = 2;
+
+template <int DT, bool ALIGNED, bool FULL>
 __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a) {
     grid_dependency_begin();
     using E = Elem<DT>;
@@ -492,6 +500,19 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
     // per-segment state; cnt, theta and seg_valid are warp-uniform
     float mu = -INFINITY;
     unsigned long long sum2 = 0ull;  // the running sum as a pair of fp32 partial sums
+    // full support: the row's request constants, the running tempered sum
+    // (sum exp(tau - mu/T), tau = l/T correctly rounded) and the best Gumbel keys
+    float fT = 1.0f;
+    unsigned long long fseed = 0ull, foff = 0ull, sumT2 = 0ull;
+    int fpar = 0;
+    // m = 1: this thread's largest logit (first on ties) is kept out of the
+    // tempered sum and added back at the row's end unless it is the row's lead,
+    // so the tail's sum never subtracts a dominant term
+    float kx = -INFINITY;
+    int kid = -1;
+    unsigned long long gk[kGumbelKeep];
+#pragma unroll
+    for (int q = 0; q < kGumbelKeep; ++q) gk[q] = 0ull;
     unsigned long long theta = 0ull;
     int cnt = 0, seg_tiles = 0;
     int64_t seg_valid = 0;
@@ -524,9 +545,22 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
         else
             s_pre.ps = 0.0f;  // reported as an internal error at the segment's end
     };
-    auto seg_begin = [&]() {
+    auto seg_begin = [&](int64_t r) {
         mu = -INFINITY;
         sum2 = 0ull;
+        if constexpr (FULL) {
+            const int b = (int)(r / a.F), f = (int)(r % a.F);
+            fT = __ldg(a.T + b);
+            fseed = __ldg(reinterpret_cast<const unsigned long long*>(a.seed) + b);
+            foff = __ldg(reinterpret_cast<const unsigned long long*>(a.offset) + b);
+            fpar = (a.d == 1) ? 0 : __ldcg(a.tree.frontier + (int64_t)b * K + f);
+            if (fpar < 0 || fpar >= n.G1) fpar = 0;  // reported at the row's end
+            sumT2 = 0ull;
+            kx = -INFINITY;
+            kid = -1;
+#pragma unroll
+            for (int q = 0; q < kGumbelKeep; ++q) gk[q] = 0ull;
+        }
         seg_valid = 0;
         cnt = 0;
         for (int i = tid; i < (kFineBins + kCoarseBins) / 4; i += kXThreads)
@@ -554,6 +588,55 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
 #pragma unroll
             for (int j = 1; j < kVPT; ++j) t = f2_add(t, W::vexp2(v[j], c2, n2));
             sum2 = f2_add(sum2, t);
+        }
+    };
+    // full support, per element: tau = l/T, the tempered sum at the running
+    // maximum mu/T, and the Gumbel key tau + g (Philox tag 1, node = the parent,
+    // draw = token id) against this thread's kept keys
+    auto tile_full = [&](const uint4 (&v)[kVPT], int e0, float mu_prev) {
+        const float mT = __fdiv_rn(mu, fT);
+        if (mu_prev != mu && mu_prev != -INFINITY) {
+            const float rs = fast_exp2(__fsub_rn(__fdiv_rn(mu_prev, fT), mT) * kLog2e);
+            sumT2 = f2_mul(sumT2, f2_pack(rs, rs));
+        }
+        if (mu == -INFINITY) return;
+        const float nmc = -mT * kLog2e;
+#pragma unroll
+        for (int j = 0; j < kVPT; ++j) {
+            const int ev = e0 + (j * kXThreads + tid) * VEC;  // first element of this vector
+            float tsum0 = 0.0f, tsum1 = 0.0f;
+#pragma unroll
+            for (int h = 0; h < VEC / 4; ++h) {
+                const uint4 rnd = philox_block(fseed, foff, kTagSample, fpar, (uint64_t)((ev >> 2) + h));
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const float x = E::value(E::raw(v[j], 4 * h + i));
+                    const float tau = __fdiv_rn(x, fT);
+                    float tv;
+                    if (m == 1 && x > kx) {  // the new largest stays out; the one it displaces joins
+                        tv = (kx > -INFINITY) ? fast_exp2(fmaf(__fdiv_rn(kx, fT), kLog2e, nmc)) : 0.0f;
+                        kx = x;
+                        kid = ev + 4 * h + i;
+                    } else {
+                        tv = fast_exp2(fmaf(tau, kLog2e, nmc));
+                    }
+                    if (i & 1) tsum1 += tv; else tsum0 += tv;
+                    const float key = __fadd_rn(tau, gumbel(u01(word_of(rnd, i))));
+                    if (key > -INFINITY) {
+                        const unsigned long long pk = make_key(ord_f32(key), ev + 4 * h + i);
+                        if (pk > gk[kGumbelKeep - 1]) {  // insert, keeping gk sorted descending
+                            unsigned long long c = pk;
+#pragma unroll
+                            for (int q = 0; q < kGumbelKeep; ++q) {
+                                const unsigned long long hi = c > gk[q] ? c : gk[q];
+                                c = c > gk[q] ? gk[q] : c;
+                                gk[q] = hi;
+                            }
+                        }
+                    }
+                }
+            }
+            sumT2 = f2_add(sumT2, f2_pack(tsum0, tsum1));
         }
     };
     // The bound theta.  On the first step of a segment: every warp's kb-th
@@ -759,23 +842,72 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
         const int64_t eidx = (a.d == 1) ? 0 : 1 + (int64_t)(a.d - 2) * K + f;
         const int64_t g0 = depth_base(K, a.d) + (int64_t)f * (K + 1);
 
-        // tempered tail q~ = softmax(l / T) over support ranks m+1..S; Y by Gumbel-max
-        const float tau = (tid < TL) ? __fdiv_rn(e2.l[m + tid], T) : -INFINITY;
-        const float mt = __fdiv_rn(e2.l[m], T);  // the support is sorted: rank m is the tail's maximum
-        const FF st = red_sum_ff<kXWarps>(FF{(tid < TL && mt > -INFINITY) ? expf(tau - mt) : 0.0f, 0.0f}, red, par);
-        const FF lse_tail = ff_add(ff_log(st), mt);
-        unsigned long long pack = 0ull;
-        if (tid < TL) {
-            e2.q[tid] = expf(__fsub_rn(tau, lse_tail.hi) - lse_tail.lo);
-            const float g = gumbel(uniform(seed, off, kTagSample, (int)par_g, (uint64_t)tid));
-            const float key = __fadd_rn(tau, g);
-            if (key > -INFINITY) pack = make_key(ord_f32(key), tid);
+        if constexpr (!FULL) {
+            // tempered tail q~ = softmax(l / T) over support ranks m+1..S; Y by Gumbel-max
+            const float tau = (tid < TL) ? __fdiv_rn(e2.l[m + tid], T) : -INFINITY;
+            const float mt = __fdiv_rn(e2.l[m], T);  // the support is sorted: rank m is the tail's maximum
+            const FF st = red_sum_ff<kXWarps>(FF{(tid < TL && mt > -INFINITY) ? expf(tau - mt) : 0.0f, 0.0f}, red, par);
+            const FF lse_tail = ff_add(ff_log(st), mt);
+            unsigned long long pack = 0ull;
+            if (tid < TL) {
+                e2.q[tid] = expf(__fsub_rn(tau, lse_tail.hi) - lse_tail.lo);
+                const float g = gumbel(uniform(seed, off, kTagSample, (int)par_g, (uint64_t)tid));
+                const float key = __fadd_rn(tau, g);
+                if (key > -INFINITY) pack = make_key(ord_f32(key), tid);
+            }
+            const unsigned long long bestp = red_max_u64<kXWarps>(pack, red, par);
+            if (tid == 0) {
+                e2.best = bestp ? (int)(0xFFFFFFFFu - (uint32_t)bestp) : 0;
+                e2.lse_tail = __fadd_rn(lse_tail.hi, lse_tail.lo);
+                if (!bestp) atomicOr(a.status, kStEmptyRow);
+            }
+        } else {
+            // full support: the tempered partition over V (each thread's sum at its
+            // maximum mu/T), the tail's = minus the leads; Y = the best Gumbel key
+            // that is not a lead (merged over the block, m+1 rounds)
+            float MT;
+            const float mT = __fdiv_rn(mu, fT);
+            float sT = f2_fold(sumT2);
+            if (m == 1 && kid >= 0 && kid != e2.id[0])  // kept out, and not the lead: it belongs to the tail
+                sT += fast_exp2(fmaf(__fdiv_rn(kx, fT), kLog2e, -mT * kLog2e));
+            const FF ST = red_partition<kXWarps>(mT, sT, kLog2e, MT, red, par);  // the tail's sum
+            for (int q = 0; q <= m; ++q) {
+                const unsigned long long bq = red_max_u64<kXWarps>(gk[0], red, par);
+                if (bq != 0ull && gk[0] == bq) {
+#pragma unroll
+                    for (int i = 0; i + 1 < kGumbelKeep; ++i) gk[i] = gk[i + 1];
+                    gk[kGumbelKeep - 1] = 0ull;
+                }
+                if (tid == 0) e2.gk[q] = bq;
+            }
+            if (tid == 0) {
+                int yid = -1;
+                for (int q = 0; q <= m && yid < 0; ++q) {
+                    if (!e2.gk[q]) break;
+                    const int id = (int)(0xFFFFFFFFu - (uint32_t)e2.gk[q]);
+                    bool lead = false;
+                    for (int i = 0; i < m; ++i) lead |= (e2.id[i] == id);
+                    if (!lead) yid = id;
+                }
+                const FF lse_tail = ff_add(ff_log(ST), MT);
+                e2.lse_tail = __fadd_rn(lse_tail.hi, lse_tail.lo);
+                e2.yid = yid;
+                e2.best = -1;
+                e2.qy = 0.0f;
+                if (yid < 0) {
+                    atomicOr(a.status, kStEmptyRow);
+                } else {
+                    const char* rowp = a.logits + r * a.row_stride_bytes;
+                    const float tauy = __fdiv_rn(E::value(E::load_scalar(rowp, yid)), T);
+                    e2.qy = expf(__fsub_rn(tauy, lse_tail.hi) - lse_tail.lo);
+                    for (int j = m; j < S; ++j)
+                        if (e2.id[j] == yid) e2.best = j;
+                }
+            }
         }
-        const unsigned long long bestp = red_max_u64<kXWarps>(pack, red, par);
         if (tid == 0) {
-            e2.best = bestp ? (int)(0xFFFFFFFFu - (uint32_t)bestp) : 0;
             if (e2.bad) atomicOr(a.status, kStInternal);
-            if (!bestp || !(e2.l[m] > -INFINITY)) atomicOr(a.status, kStEmptyRow);
+            if (!(e2.l[m] > -INFINITY)) atomicOr(a.status, kStEmptyRow);
             if (!(T > 0.0f) || isinf(T)) atomicOr(a.status, kStBadTemperature);
             // construction probability of Y (Sec. 3.2): min{q0(x_m), z}, never below
             // q0(x_{m+1}); m = 0: min(1, q0(x_1) + eps)
@@ -808,20 +940,31 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
         const int best = e2.best;
         if (tid <= K) {
             const int j = tid;
-            int rank;
+            int rank, tok;
             float lpj, qv = 0.0f;
             uint8_t st8;
             if (j < m) {
                 rank = j; lpj = e2.lq0[j]; st8 = kSlotLead;
+                tok = e2.id[rank];
             } else if (j == m) {
-                rank = m + best; lpj = e2.lp; st8 = kSlotSampled; qv = e2.q[best];
+                lpj = e2.lp; st8 = kSlotSampled;
+                if constexpr (FULL) {
+                    tok = e2.yid; qv = e2.qy;
+                } else {
+                    rank = m + best; qv = e2.q[best]; tok = e2.id[rank];
+                }
             } else {
                 const int qf = j - m - 1;
-                rank = m + qf + (qf >= best ? 1 : 0); lpj = e2.lq0[rank]; st8 = kSlotFill;
+                if constexpr (FULL)
+                    rank = m + qf + ((best >= 0 && m + qf >= best) ? 1 : 0);
+                else
+                    rank = m + qf + (qf >= best ? 1 : 0);
+                lpj = e2.lq0[rank]; st8 = kSlotFill;
+                tok = e2.id[rank];
             }
             const float ps = s_pre.ps;
             const int64_t g = nb + g0 + j;
-            a.tree.token[g] = e2.id[rank];
+            a.tree.token[g] = tok;
             a.tree.parent[g] = (int32_t)par_g;
             a.tree.log_proxy[g] = lpj;
             a.tree.score[g] = __fadd_rn(ps, lpj);
@@ -833,7 +976,10 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             a.tree.tail_ids[q0 + tid] = e2.id[m + tid];
             a.tree.tail_q[q0 + tid] = e2.q[tid];
         }
-        if (tid == 0) a.tree.lse1[(int64_t)b * n.E + eidx] = lse1;
+        if (tid == 0) {
+            a.tree.lse1[(int64_t)b * n.E + eidx] = lse1;
+            if (a.tree.lse_tail) a.tree.lse_tail[(int64_t)b * n.E + eidx] = e2.lse_tail;
+        }
 
         // ---- last row of the request: the K best depth-d nodes become the frontier ----
         if (!arrive_last(a.req_ticket + b, (unsigned)a.F, bs)) return;
@@ -901,12 +1047,14 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             }
             if (seg_first) {
                 prefetch_row(r);
-                seg_begin();
+                seg_begin(r);
             } else if (tid == 0 && s_pre.stage == 1) {
                 prefetch_parent(r);
             }
             float vm[kVPT];
+            const float mu_prev = mu;
             tile_sum(v, vm);
+            if constexpr (FULL) tile_full(v, e0, seg_first ? -INFINITY : mu_prev);
             refresh(seg_first);
             seg_valid += ne;
             tile_candidates(v, vm, e0);
@@ -915,14 +1063,19 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
     }
 }
 
-cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, int grid, size_t smem, cudaStream_t s) {
+cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, bool full, int grid, size_t smem,
+                          cudaStream_t s) {
     auto go = [&](auto kern) {
         cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (err != cudaSuccess) return err;
         return launch_dependent(kern, dim3(grid), dim3(kXThreads), smem, s, a);
     };
-    if (dtype == 1) return aligned ? go(expand_kernel<1, true>) : go(expand_kernel<1, false>);
-    return aligned ? go(expand_kernel<0, true>) : go(expand_kernel<0, false>);
+    if (full) {
+        if (dtype == 1) return aligned ? go(expand_kernel<1, true, true>) : go(expand_kernel<1, false, true>);
+        return aligned ? go(expand_kernel<0, true, true>) : go(expand_kernel<0, false, true>);
+    }
+    if (dtype == 1) return aligned ? go(expand_kernel<1, true, false>) : go(expand_kernel<1, false, false>);
+    return aligned ? go(expand_kernel<0, true, false>) : go(expand_kernel<0, false, false>);
 }
 
 size_t expand_keys_bytes(int max_segments, int support) {

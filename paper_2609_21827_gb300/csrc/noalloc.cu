@@ -103,8 +103,8 @@ extern "C" int rheo_verify_static(const rheo_config* cfg, const void* logits, in
                                   const float* temperature, const uint64_t* seed, const uint64_t* offset,
                                   const rheo_tree* tree, const rheo_pruned* pruned, const rheo_verify_out* out,
                                   int32_t* status, rheo_stream_t stream) {
-    if (!config_ok(cfg) || !logits || row_stride < cfg->vocab || !temperature || !seed || !offset ||
-        !buffers_ok(tree, pruned, out))
+    if (!config_ok(cfg) || cfg->support == 0 || !logits || row_stride < cfg->vocab || !temperature || !seed ||
+        !offset || !buffers_ok(tree, pruned, out))
         return RHEO_EINVAL;
     const StaticLayout L = static_layout(*cfg);
     if (L.total > kStaticScratchBytes) return RHEO_ETOOLARGE;

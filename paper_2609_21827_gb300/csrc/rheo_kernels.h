@@ -17,6 +17,7 @@ struct TreePtrs {
     int32_t* tail_ids;
     float* tail_q;
     float* lse1;
+    float* lse_tail;   // [B, E] or null (sparse support); required with full support
 };
 
 struct PrunedPtrs {
@@ -31,6 +32,7 @@ struct PrunedPtrs {
 
 struct Dims {
     int B, V, K, m, S, D, N;
+    int full;    // full support: S = K+1 ranks selected, the sampled token drawn over V
     int TL;      // S - m
     int GW;      // gathered logits per verify row: (K+1) + TL
     int chunks;  // chunks per row
@@ -130,7 +132,8 @@ cudaError_t launch_dependent(void (*kern)(P...), dim3 grid, dim3 block, size_t s
 // aligned: every row starts on a 16-byte boundary, so rows are read with
 // 16-byte vector loads (a row's ragged end element-wise); otherwise element-wise.
 // whole: every CTA's tiles lie in one row (the two halves are streamed side by side)
-cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, int grid, size_t smem, cudaStream_t s);
+cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, bool full, int grid, size_t smem,
+                          cudaStream_t s);
 cudaError_t launch_prune(const PruneArgs& a, int batch, size_t smem, cudaStream_t s);
 cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid, cudaStream_t s);
 size_t expand_keys_bytes(int max_segments, int support);

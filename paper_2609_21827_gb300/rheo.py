@@ -40,7 +40,7 @@ _VP = ctypes.c_void_p
 
 class _Tree(ctypes.Structure):
     _fields_ = [(n, _VP) for n in ("token", "parent", "log_proxy", "score", "qtilde", "slot", "frontier",
-                                   "tail_ids", "tail_q", "lse1")]
+                                   "tail_ids", "tail_q", "lse1", "lse_tail")]
 
 
 class _Pruned(ctypes.Structure):
@@ -147,7 +147,7 @@ class Tree:
 
     def __init__(self, cfg: Config, device="cuda"):
         G1, E, _ = cfg.sizes()
-        B, TL = cfg.batch, cfg.support - cfg.m
+        B, TL = cfg.batch, (0 if cfg.support == 0 else cfg.support - cfg.m)
         i32, f32 = torch.int32, torch.float32
         self.token = torch.full((B, G1), -1, dtype=i32, device=device)
         self.parent = torch.full((B, G1), -1, dtype=i32, device=device)
@@ -159,6 +159,7 @@ class Tree:
         self.tail_ids = torch.zeros((B, E, TL), dtype=i32, device=device)
         self.tail_q = torch.zeros((B, E, TL), dtype=f32, device=device)
         self.lse1 = torch.zeros((B, E), dtype=f32, device=device)
+        self.lse_tail = torch.zeros((B, E), dtype=f32, device=device)
 
     def c(self) -> _Tree:
         return _Tree(*[getattr(self, n).data_ptr() for n, _ in _Tree._fields_])

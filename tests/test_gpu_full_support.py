@@ -1,0 +1,103 @@
+"""GPU parity of full support (support = 0: the sampled token over the whole
+vocabulary; App. B, Table tab:sparse_support, row Full) against the oracle.
+
+Expansion and prune on both sides from the same seeded draft rows: tokens,
+parents, slots, frontiers and pruned trees bit-exact, scores / log proxies /
+lse1 / lse_tail within the log-domain tolerance, q~(Y) within rtol 1e-5; a
+request whose first difference sits at a Gumbel or frontier decision with an
+oracle margin below 1e-6 counts as an explained near-tie flip.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_21827_gb300 import build, rheo, synth
+import parity_harness as ph
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    build.build()
+    import oracle
+    oracle.build()
+
+
+def _W(name, **kw):
+    base = dict(name=name, batch=6, vocab=3000, depth=3, K=4, budget=12, dtype="f32", zipf_s=1.1,
+                sigma_draft=0.5, sigma_target=0.5, temperatures=(1.0,), seed=8181)
+    base.update(kw)
+    return synth.Workload(**base)
+
+
+CASES = [
+    _W("small"),
+    _W("v40_m0", vocab=40, K=3, m=0, depth=2, budget=6, batch=16),
+    _W("m1_bf16", vocab=5000, K=5, m=1, depth=3, budget=14, dtype="bf16", temperatures=(0.6, 1.3)),
+    _W("ragged", vocab=20011, K=6, m=1, depth=3, budget=20, dtype="bf16", temperatures=(0.8,)),
+    _W("low_T", vocab=2000, K=4, depth=3, budget=10, temperatures=(0.05,)),
+]
+
+
+def _cfg(w):
+    return rheo.Config(batch=w.batch, vocab=w.vocab, K=w.K, depth=w.depth, budget=w.budget, m=w.m, support=0,
+                       dtype=w.dtype)
+
+
+def _run(w, reqs):
+    import oracle
+    cfg = _cfg(w)
+    draft = synth.make_draft_inputs(w, device="cuda")
+    tree, pr, ws = rheo.Tree(cfg), rheo.Pruned(cfg), rheo.Workspace(cfg)
+    for d in range(1, cfg.depth + 1):
+        rheo.expand(cfg, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tree, ws)
+    rheo.prune(cfg, tree, pr, ws)
+    assert rheo.status(cfg, ws) == 0
+    ocfg = oracle.Config(B=len(reqs), V=w.vocab, K=w.K, m=w.m, S=0, D=w.depth, N=w.budget, eps=cfg.eps)
+    ot = oracle.Tree(ocfg)
+    T = draft.temperature.cpu().numpy()[reqs]
+    seed, off = ph.u64(draft.seed)[reqs], ph.u64(draft.offset)[reqs]
+    for d in range(1, w.depth + 1):
+        oracle.expand(ocfg, d, draft.rows[d - 1][reqs].float().cpu().numpy(), T, seed, off, ot)
+    op = oracle.prune(ocfg, ot)
+    g = {k: getattr(tree, k).cpu().numpy() for k in ("token", "parent", "slot", "score", "log_proxy", "qtilde",
+                                                      "lse1", "lse_tail")}
+    gp = {k: getattr(pr, k).cpu().numpy() for k in ("gen_id", "parent", "first_child", "n_child", "sampled_child")}
+    explained = 0
+    for j, b in enumerate(reqs):
+        same = (np.array_equal(g["token"][b], ot.token[j]) and np.array_equal(g["parent"][b], ot.parent[j])
+                and np.array_equal(g["slot"][b], ot.slot[j]) and np.array_equal(gp["gen_id"][b], op.gen_id[j]))
+        if not same:
+            gap = min(float(np.min(ot.gap_sample[j])), float(np.min(ot.gap_frontier[j])), float(op.gap_prune[j]))
+            assert gap < ph.GAP, f"{w.name} request {b}: trees differ, oracle margin {gap}"
+            explained += 1
+            continue
+        for k in ("parent", "first_child", "n_child", "sampled_child"):
+            np.testing.assert_array_equal(gp[k][b], getattr(op, k)[j], err_msg=k)
+        for k in ("score", "log_proxy", "lse1", "lse_tail"):
+            a, o = g[k][b].astype(np.float64), getattr(ot, k)[j].astype(np.float64)
+            assert np.all(np.abs(a - o) <= ph.LOG_ATOL + ph.RTOL * np.abs(o)), (w.name, b, k)
+        a, o = g["qtilde"][b].astype(np.float64), ot.qtilde[j].astype(np.float64)
+        assert np.all(np.abs(a - o) <= ph.ATOL + ph.RTOL * np.abs(o)), (w.name, b, "qtilde")
+    return explained
+
+
+@pytest.mark.parametrize("w", CASES, ids=[w.name for w in CASES])
+def test_full_support_tree_parity(w):
+    reqs = list(range(w.batch))
+    assert _run(w, reqs) <= 1
+
+
+def test_full_support_requires_m_at_most_one():
+    import ctypes
+    cfg = rheo.Config(batch=2, vocab=1000, K=4, depth=2, budget=8, m=2, support=0, dtype="f32")
+    sz = ctypes.c_size_t()
+    assert rheo.lib().rheo_sizes(ctypes.byref(cfg.c()), None, None, ctypes.byref(sz)) == rheo.RHEO_EINVAL
+
+
+def test_full_support_tree_parity_qwen3_size():
+    w = synth.WORKLOADS["qwen3_batch"]
+    assert _run(w, [1, 12]) <= 1

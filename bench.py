@@ -467,6 +467,58 @@ def main(argv=None):
     synthetic_lm = {"vocab": 64, "k": 2, "K": 8, "depth": 6, "budget": 40, "sequences": 1024, "cycles": 6,
                     "tau": tau, "host_ms_per_cycle": lm_ms / 8}
 
+    # full support (App. B, Table tab:sparse_support, row Full): the same
+    # workload with the sampled token drawn over the whole vocabulary; a graph
+    # of its 12 launches timed like the main step, plus per-call times
+    cfg_f = rheo.Config(batch=w.batch, vocab=w.vocab, K=w.K, depth=w.depth, budget=w.budget, m=w.m, support=0,
+                        dtype=w.dtype)
+    tf, pf, wf = rheo.Tree(cfg_f, device), rheo.Pruned(cfg_f, device), rheo.Workspace(cfg_f, device)
+    of = rheo.VerifyOut(cfg_f, row_lse=False, device=device)
+    fr_f = []
+    for d in range(1, D + 1):
+        rheo.expand(cfg_f, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tf, wf)
+        if d < D:
+            fr_f.append(tf.frontier.clone())
+    rheo.prune(cfg_f, tf, pf, wf)
+    tgt_f = synth.target_rows(w, draft, fr_f, pf.gen_id)
+
+    def step_f(s_, marks=None):
+        for d in range(1, D + 1):
+            rheo.expand(cfg_f, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tf, wf, s_)
+        if marks:
+            marks[0].record(s_)
+        rheo.prune(cfg_f, tf, pf, wf, s_)
+        if marks:
+            marks[1].record(s_)
+        rheo.verify_full(cfg_f, tgt_f, draft.rows, draft.temperature, draft.seed, draft.offset, tf, pf, of, wf, s_)
+
+    g_f = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        step_f(stream)
+        stream.synchronize()
+        with torch.cuda.graph(g_f, stream=stream):
+            step_f(stream)
+        for _ in range(3):
+            g_f.replay()
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n_f = max(20, min(200, args.steps))
+        f0.record(stream)
+        for _ in range(n_f):
+            g_f.replay()
+        f1.record(stream)
+        stream.synchronize()
+        ms_f = f0.elapsed_time(f1) / n_f
+        mk = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        mk[0].record(stream)
+        step_f(stream, marks=(mk[1], mk[2]))
+        mk[3].record(stream)
+        stream.synchronize()
+    assert rheo.status(cfg_f, wf, stream) == 0
+    full_support = {"tree_steps_per_s": 1e3 / ms_f, "ms_per_step": ms_f,
+                    "expand_ms": mk[0].elapsed_time(mk[1]), "prune_ms": mk[1].elapsed_time(mk[2]),
+                    "verify_ms": mk[2].elapsed_time(mk[3]),
+                    "note": "eager per-call times; the step time is the CUDA graph of its 12 launches"}
+
     # end to end through the public API with host buffers: H2D of every input, D2H of the results
     e2e = None
     if rank == 0 or world > 1:
@@ -551,6 +603,7 @@ def main(argv=None):
                     "tree_attention_us": attn_us,
                     "verify_variants": variants,
                     "synthetic_lm": synthetic_lm,
+                    "full_support": full_support,
                     "tree_attention_bytes": w.batch * (w.budget + 1) * ((w.budget + 1) + 4 + 4 * (w.depth + 1) + 12)},
         "clocks": clocks,
         "gpu_launches": args.steps * (D + 4),  # D expand, 1 prune, 3 verify (prep, stream, residual)

@@ -185,6 +185,22 @@ int rheo_verify_variant(const rheo_config* cfg, int32_t variant, const void* tar
                         const rheo_tree* tree, const rheo_pruned* pruned, const rheo_verify_out* out,
                         void* workspace, rheo_stream_t stream);
 
+/* Verification of a tree built with full support (cfg.support = 0; App. B,
+ * Table tab:sparse_support, row Full), Algorithm 1 as rheo_verify.  With no
+ * tail lists, q~ over the whole vocabulary is re-derived from the draft rows:
+ * draft_logits is a host array of cfg.depth device pointers, entry d-1 the
+ * [B, F_d, V] draft logits passed to rheo_expand at depth d (row b*F_d + f at
+ * element (b*F_d + f)*draft_row_stride); they must be unchanged since the
+ * expansion, and the workspace must be the one the expansions used (it holds
+ * the tails' log-partitions).  At a node whose sampled child survived:
+ * q~(v) = exp(l_d(v)/T - lse_tail) off the lead, 0 at the lead,
+ * M = 1 - sum_V min(p, q~), r^ = max(0, p - q~).  Requires depth <= 32.
+ * Other arguments, outputs and errors as rheo_verify. */
+int rheo_verify_full(const rheo_config* cfg, const void* target_logits, int64_t row_stride,
+                     const void* const* draft_logits, int64_t draft_row_stride, const float* temperature,
+                     const uint64_t* seed, const uint64_t* offset, const rheo_tree* tree, const rheo_pruned* pruned,
+                     const rheo_verify_out* out, void* workspace, rheo_stream_t stream);
+
 /* Verification for callers that cannot allocate device memory where they
  * verify (code handed only fixed input/output buffers by a host framework,
  * runtimes whose device memory is partitioned up front, loops that must not

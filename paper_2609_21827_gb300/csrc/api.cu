@@ -46,7 +46,7 @@ bool valid(const rheo_config* c) {
 }
 
 struct Layout {
-    size_t status, ex_row_ticket, ex_req_ticket, ex_mu, ex_sum, ex_keys;
+    size_t status, ex_row_ticket, ex_req_ticket, ex_mu, ex_sum, ex_keys, ex_ltail;
     size_t v_mu, v_sum, v_row_ticket, v_hdr, v_child, v_tids, v_tq, v_cx, v_tx, v_coin, v_table, v_rhat, r_best,
         r_ticket;
     size_t total;
@@ -67,6 +67,7 @@ Layout layout(const rheo_config& c) {
     L.ex_mu = take(sizeof(float) * B * F * P);
     L.ex_sum = take(2 * sizeof(float) * B * F * P);
     L.ex_keys = take(sizeof(unsigned long long) * B * F * P * S);
+    L.ex_ltail = take(2 * sizeof(float) * B * expansions_per_request(c));
     L.v_mu = take(sizeof(float) * B * NP * VC);
     L.v_sum = take(2 * sizeof(float) * B * NP * VC);
     L.v_row_ticket = take(sizeof(unsigned) * B * NP);
@@ -185,6 +186,7 @@ extern "C" int rheo_expand(const rheo_config* cfg, int32_t d, const void* logits
     a.seg_mu = at<float>(ws, L.ex_mu);
     a.seg_sum = at<float>(ws, L.ex_sum);
     a.seg_keys = at<unsigned long long>(ws, L.ex_keys);
+    a.lse_tail_ff = at<float>(ws, L.ex_ltail);
     const int tpr = tiles_per_row(*cfg);
     const int64_t rows = (int64_t)cfg->batch * a.F;
     const int sms = sm_count();
@@ -293,6 +295,68 @@ extern "C" int rheo_verify_variant(const rheo_config* cfg, int32_t variant, cons
     const int grid = verify_stream_grid(sm_count(), chunks);
     a.units = verify_stream_units(grid, chunks);
     return launch_verify(a, cfg->dtype, rows_aligned(logits, row_stride, *cfg), grid, (cudaStream_t)stream) ==
+                   cudaSuccess
+               ? RHEO_OK
+               : RHEO_ELAUNCH;
+}
+
+extern "C" int rheo_verify_full(const rheo_config* cfg, const void* logits, int64_t row_stride,
+                                const void* const* draft_logits, int64_t draft_row_stride, const float* temperature,
+                                const uint64_t* seed, const uint64_t* offset, const rheo_tree* tree,
+                                const rheo_pruned* pruned, const rheo_verify_out* out, void* ws, rheo_stream_t stream) {
+    if (!cfg || cfg->support != 0 || cfg->depth > kMaxFullDepth || !draft_logits || draft_row_stride < cfg->vocab)
+        return RHEO_EINVAL;
+    for (int d = 0; d < cfg->depth; ++d)
+        if (!draft_logits[d]) return RHEO_EINVAL;
+    if (!valid(cfg) || !logits || row_stride < cfg->vocab || !temperature || !seed || !offset || !tree_ok(tree, *cfg) ||
+        !pruned_ok(pruned) || !out || !out->accepted_len || !out->accepted_tokens || !out->accepted_nodes ||
+        !out->bonus_token || !ws)
+        return RHEO_EINVAL;
+    const Layout L = layout(*cfg);
+    VerifyArgs a;
+    a.n = dims(*cfg);
+    a.variant = kVerifyRheo;
+    bool draft_aligned = (draft_row_stride * elem_size(*cfg)) % 16 == 0;
+    for (int d = 0; d < cfg->depth; ++d) {
+        a.draft[d] = static_cast<const char*>(draft_logits[d]);
+        draft_aligned = draft_aligned && (reinterpret_cast<uintptr_t>(draft_logits[d]) % 16 == 0);
+    }
+    a.draft_row_stride_bytes = draft_row_stride * elem_size(*cfg);
+    a.lse_tail_ff = at<float>(ws, L.ex_ltail);
+    a.logits = static_cast<const char*>(logits);
+    a.row_stride_bytes = row_stride * elem_size(*cfg);
+    a.T = temperature;
+    a.seed = seed;
+    a.offset = offset;
+    a.tree = tree_ptrs(tree);
+    a.pr = pruned_ptrs(pruned);
+    a.accepted_len = out->accepted_len;
+    a.accepted_tokens = out->accepted_tokens;
+    a.accepted_nodes = out->accepted_nodes;
+    a.bonus_token = out->bonus_token;
+    a.row_lse = out->row_lse;
+    a.status = at<unsigned>(ws, L.status);
+    a.seg_mu = at<float>(ws, L.v_mu);
+    a.seg_sum = at<float>(ws, L.v_sum);
+    a.row_ticket = at<unsigned>(ws, L.v_row_ticket);
+    a.rec_hdr = at<int>(ws, L.v_hdr);
+    a.rec_child = at<int>(ws, L.v_child);
+    a.rec_tids = at<int>(ws, L.v_tids);
+    a.rec_tq = at<float>(ws, L.v_tq);
+    a.rec_cx = at<float>(ws, L.v_cx);
+    a.rec_tx = at<float>(ws, L.v_tx);
+    a.rec_coin = at<float>(ws, L.v_coin);
+    a.table = at<float>(ws, L.v_table);
+    a.rhat_tail = at<float>(ws, L.v_rhat);
+    a.res_best = at<unsigned long long>(ws, L.r_best);
+    a.res_ticket = at<unsigned>(ws, L.r_ticket);
+    const int64_t NP = cfg->budget + 1;
+    a.n.chunks = verify_chunks_per_row(cfg->dtype == RHEO_BF16 ? 1 : 0, cfg->vocab);
+    const int64_t chunks = (int64_t)cfg->batch * NP * a.n.chunks;
+    const int grid = verify_stream_grid(sm_count(), chunks);
+    a.units = verify_stream_units(grid, chunks);
+    return launch_verify_full(a, cfg->dtype, rows_aligned(logits, row_stride, *cfg), draft_aligned, grid,
+                              (cudaStream_t)stream) ==
                    cudaSuccess
                ? RHEO_OK
                : RHEO_ELAUNCH;

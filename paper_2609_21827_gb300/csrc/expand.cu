@@ -891,6 +891,9 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
                 }
                 const FF lse_tail = ff_add(ff_log(ST), MT);
                 e2.lse_tail = __fadd_rn(lse_tail.hi, lse_tail.lo);
+                const int64_t ei = (a.d == 1) ? 0 : 1 + (int64_t)(a.d - 2) * K + f;
+                a.lse_tail_ff[2 * ((int64_t)b * n.E + ei)] = lse_tail.hi;
+                a.lse_tail_ff[2 * ((int64_t)b * n.E + ei) + 1] = lse_tail.lo;
                 e2.yid = yid;
                 e2.best = -1;
                 e2.qy = 0.0f;

@@ -56,6 +56,7 @@ struct ExpandArgs {
     float* seg_mu;                  // [B*F*tiles_per_row]
     float* seg_sum;                 // [B*F*tiles_per_row*2] float-float partition sums
     unsigned long long* seg_keys;   // [B*F*tiles_per_row*S]
+    float* lse_tail_ff;             // [B*E*2] full support: the tail's log-partition as float-float
 };
 
 struct PruneArgs {
@@ -76,6 +77,7 @@ struct TreeAttnArgs {
 };
 
 enum : int { kVerifyRheo = 0, kVerifyRrsw = 1, kVerifyOneHot = 2 };
+constexpr int kMaxFullDepth = 32;  // depth limit of full-support verification
 
 struct VerifyArgs {
     Dims n;                         // n.chunks: 2 KB chunks per target row
@@ -108,6 +110,12 @@ struct VerifyArgs {
     float* rhat_tail;               // [B*(N+1)*TL]
     unsigned long long* res_best;   // [B*3]
     unsigned* res_ticket;           // [B]
+    // full support: the draft rows of the expanded nodes (depth d: [B, F_d, V]
+    // rows at draft[d-1] + (b*F_d + f) * draft_row_stride_bytes) and the tails'
+    // log-partitions written by the expansions
+    const char* draft[kMaxFullDepth] = {};
+    int64_t draft_row_stride_bytes = 0;
+    const float* lse_tail_ff = nullptr;  // [B*E*2]
 };
 
 // Launch with the programmatic stream serialization attribute: the kernel may
@@ -136,6 +144,8 @@ cudaError_t launch_expand(const ExpandArgs& a, int dtype, bool aligned, bool ful
                           cudaStream_t s);
 cudaError_t launch_prune(const PruneArgs& a, int batch, size_t smem, cudaStream_t s);
 cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid, cudaStream_t s);
+cudaError_t launch_verify_full(const VerifyArgs& a, int dtype, bool aligned, bool draft_aligned, int grid,
+                               cudaStream_t s);
 size_t expand_keys_bytes(int max_segments, int support);
 size_t expand_smem_bytes(int max_segments, int support);
 int expand_tile_elems(int dtype);

@@ -369,6 +369,8 @@ __device__ __noinline__ void finalize_row(const VerifyArgs& a, int64_t r, WarpRo
         if (!(lse.hi > -INFINITY)) atomicOr(a.status, kStEmptyRow);
         if ((r % NP) == 0 && (!(T > 0.0f) || isinf(T))) atomicOr(a.status, kStBadTemperature);
     }
+    // full support: q~ lives in the draft row; full_overlap_kernel decides such rows
+    if (a.n.full && sc >= 0) return;
     // r^ over the tail and the overlap sum of min(p, q~) (sampled child survived)
     const int variant = a.variant;
     FF ov{0.0f, 0.0f};
@@ -541,7 +543,11 @@ __device__ __forceinline__ unsigned long long pack_key(float key, int64_t id) {
     return ((unsigned long long)ord_f32(key) << 32) | (0xFFFFFFFFu - (uint32_t)id);
 }
 
-template <int DT, bool ALIGNED>
+// Full support (FULL): every token but the lead belongs to the tail, so after a
+// rejection the key of each token outside the candidates is log r^ + g with
+// r^ = max(0, p - q~), q~ = exp(l_d/T - lse_tail) read off the stopping node's
+// draft row (DALIGNED: that row is 16-byte aligned); the lead keeps log p + g.
+template <int DT, bool ALIGNED, bool FULL = false, bool DALIGNED = false>
 __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) {
     grid_dependency_begin();
     using E = Elem<DT>;
@@ -599,6 +605,7 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     const float* tu = a.table + rowg * TW;
     const int use_tail = (int)__ldcg(tu + 5);
     const float lse = __ldcg(tu + 3);
+    const FF lse_ff{lse, __ldcg(tu + 4)};
     const float T = a.T[b];
     const uint64_t seed = a.seed[b], off = a.offset[b];
     // the stopping row's record: children and (after a rejection) its tail
@@ -609,6 +616,20 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     const int32_t* tids = a.rec_tids + rowg * TL;
     const char* row = a.logits + rowg * a.row_stride_bytes;
     const int64_t e_lo = (int64_t)k * kResChunk;
+    // full support after a rejection: the stopping node's draft row, tail
+    // log-partition and lead
+    const char* drow = nullptr;
+    FF lt{0.0f, 0.0f};
+    int lead = -1;
+    if (FULL && use_tail) {
+        const int sc = __ldcg(hdr + 2);
+        const int gs = a.pr.gen_id[pb + (sc >= 0 ? sc : 0)];
+        const int e = parent_expansion_of(K, gs);
+        const int dd = (e == 0) ? 1 : 2 + (e - 1) / K, f = (e == 0) ? 0 : (e - 1) % K;
+        drow = a.draft[dd - 1] + ((int64_t)b * (dd == 1 ? 1 : K) + f) * a.draft_row_stride_bytes;
+        lt = FF{__ldcg(a.lse_tail_ff + 2 * ((int64_t)b * n.E + e)), __ldcg(a.lse_tail_ff + 2 * ((int64_t)b * n.E + e) + 1)};
+        lead = (n.m == 1) ? a.tree.token[(int64_t)b * n.G1 + gs - 1] : -1;
+    }
 
     for (int c = tid; c < nc_ok; c += kThreads) {
         const int tok = __ldcg(rchild + 3 * c);
@@ -629,8 +650,12 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     {
         const int64_t e0 = e_lo + (int64_t)tid * kResPer;
         uint4 xv[kResPer / E::VEC];  // this thread's elements of the stopping row
+        uint4 dv[kResPer / E::VEC];  // full support: the same elements of the draft row
 #pragma unroll
-        for (int j = 0; j < kResPer / E::VEC; ++j) xv[j] = load_vec<DT, ALIGNED>(row, e0 + j * E::VEC, V);
+        for (int j = 0; j < kResPer / E::VEC; ++j) {
+            xv[j] = load_vec<DT, ALIGNED>(row, e0 + j * E::VEC, V);
+            if (FULL && drow) dv[j] = load_vec<DT, DALIGNED>(drow, e0 + j * E::VEC, V);
+        }
 #pragma unroll
         for (int h = 0; h < kResPer / 4; ++h) {
             if (e0 + 4 * h >= V) break;
@@ -644,7 +669,17 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
                 const int q = 4 * h + i;
                 const float x = E::value(E::raw(xv[q / E::VEC], q % E::VEC));
                 const float g = gumbel(u01(word_of(rnd, i)));
-                const float key = __fadd_rn(__fsub_rn(__fdiv_rn(x, T), lse), g);
+                float key;
+                if (FULL && drow && id != lead) {
+                    const float pt = exp_ff_minus(ff_div(x, T), lse_ff);
+                    const float xd = E::value(E::raw(dv[q / E::VEC], q % E::VEC));
+                    const float qt = expf(__fsub_rn(__fdiv_rn(xd, T), lt.hi) - lt.lo);
+                    const float rv = __fsub_rn(pt, qt);
+                    if (!(rv > 0.0f)) continue;
+                    key = __fadd_rn(logf(rv), g);
+                } else {
+                    key = __fadd_rn(__fsub_rn(__fdiv_rn(x, T), lse), g);
+                }
                 if (key > -INFINITY) {
                     const unsigned long long pk = pack_key(key, id);
                     best = pk > best ? pk : best;
@@ -699,6 +734,128 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
         if (!m) atomicOr(a.status, kStEmptyRow);
         a.res_best[(int64_t)b * 3] = 0ull;  // ready for the next call
     }
+}
+
+// Full support, after the stream kernel: the rows whose sampled child
+// survived.  One CTA per such row streams the target row and its node's draft
+// row side by side: p = softmax(l/T) (log-partition from the stream kernel),
+// q~ = exp(l_d/T - lse_tail) off the lead (0 at the lead), M = 1 - sum min(p,
+// q~) as float-float; then r^ = max(0, p - q~) at the children and the row's
+// decisions by Algorithm 1 (sampled child first, then the others in slot
+// order), written to the row's table as the stream kernel does for other rows.
+template <int DT, bool ALIGNED, bool DALIGNED>
+__global__ void __launch_bounds__(kThreads) full_overlap_kernel(const VerifyArgs a) {
+    grid_dependency_begin();
+    using E = Elem<DT>;
+    __shared__ Red red;
+    __shared__ float s_pc[kMaxSupport], s_rc[kMaxSupport], s_coin[kMaxSupport + 1];
+    __shared__ int s_slot[kMaxSupport];
+    const Dims& n = a.n;
+    const int tid = threadIdx.x;
+    const int64_t r = blockIdx.x;
+    const int K = n.K, NP = n.N + 1, V = n.V;
+    const int* hdr = a.rec_hdr + r * kHdr;
+    const int sc = __ldcg(hdr + 2);
+    if (sc < 0) return;  // decided by the stream kernel
+    const int nc = __ldcg(hdr + 0), fc = __ldcg(hdr + 1);
+    const float qs = __int_as_float(__ldcg(hdr + 4));
+    const int b = (int)(r / NP);
+    const int64_t pb = (int64_t)b * NP;
+    float* tab = a.table + r * table_width(K);
+    const FF lse{__ldcg(tab + 3), __ldcg(tab + 4)};
+    const float T = a.T[b];
+    const int gs = a.pr.gen_id[pb + sc];
+    const int e = parent_expansion_of(K, gs);
+    const FF lt{__ldcg(a.lse_tail_ff + 2 * ((int64_t)b * n.E + e)), __ldcg(a.lse_tail_ff + 2 * ((int64_t)b * n.E + e) + 1)};
+    const int lead = (n.m == 1) ? a.tree.token[(int64_t)b * n.G1 + gs - 1] : -1;
+    const int dd = (e == 0) ? 1 : 2 + (e - 1) / K, f = (e == 0) ? 0 : (e - 1) % K;
+    const char* drow = a.draft[dd - 1] + ((int64_t)b * (dd == 1 ? 1 : K) + f) * a.draft_row_stride_bytes;
+    const char* trow = a.logits + r * a.row_stride_bytes;
+    int par = 0;
+    FF ov{0.0f, 0.0f};
+    for (int64_t e0 = (int64_t)tid * E::VEC; e0 < V; e0 += (int64_t)kThreads * E::VEC) {
+        const uint4 tv = load_vec<DT, ALIGNED>(trow, e0, V);
+        const uint4 dv = load_vec<DT, DALIGNED>(drow, e0, V);
+#pragma unroll
+        for (int i = 0; i < E::VEC; ++i) {
+            const int64_t id = e0 + i;
+            if (id >= V) break;
+            const float pt = exp_ff_minus(ff_div(E::value(E::raw(tv, i)), T), lse);
+            const float qt = (id == lead) ? 0.0f
+                                          : expf(__fsub_rn(__fdiv_rn(E::value(E::raw(dv, i)), T), lt.hi) - lt.lo);
+            ov = ff_add(ov, fminf(pt, qt));
+        }
+    }
+    ov = red_sum_ff(ov, red, par);
+    const int nc_ok = (nc >= 0 && nc <= K + 1) ? nc : 0;
+    for (int c = tid; c < nc_ok; c += kThreads) {
+        const int* ch = a.rec_child + (r * (K + 1) + c) * 3;
+        const int tok = __ldcg(ch + 0);
+        const float pt = exp_ff_minus(ff_div(E::value(E::load_scalar(trow, tok)), T), lse);
+        const float qt = (tok == lead) ? 0.0f
+                                       : expf(__fsub_rn(__fdiv_rn(E::value(E::load_scalar(drow, tok)), T), lt.hi) - lt.lo);
+        const float dlt = __fsub_rn(pt, qt);
+        s_pc[c] = pt;
+        s_rc[c] = dlt > 0.0f ? dlt : 0.0f;
+        s_slot[c] = __ldcg(ch + 2);
+    }
+    for (int i = tid; i < K + 2; i += kThreads) s_coin[i] = __ldcg(a.rec_coin + r * (K + 2) + i);
+    __syncthreads();
+    if (tid == 0) {
+        FF M{1.0f, 0.0f};
+        int acc = -1, use_tail = 0;
+        if (sc - fc >= 0 && sc - fc < nc_ok && __fmul_rn(s_coin[0], qs) <= s_pc[sc - fc]) {
+            acc = sc;
+        } else {
+            M = ff_add(FF{1.0f, 0.0f}, ff_neg(ov));
+            use_tail = 1;
+        }
+        const FF M0 = M;
+        if (acc < 0)
+            for (int c2 = 0; c2 < nc_ok; ++c2) {
+                if (fc + c2 == sc) continue;
+                const float eta = s_coin[1 + s_slot[c2]];
+                if (ff_le(ff_mul(eta, M), s_rc[c2])) {
+                    acc = fc + c2;
+                    break;
+                }
+                M = ff_add(M, -s_rc[c2]);
+            }
+        tab[0] = M0.hi;
+        tab[1] = M0.lo;
+        tab[2] = qs;
+        tab[5] = (float)use_tail;
+        tab[6] = (float)acc;
+    }
+}
+
+cudaError_t launch_verify_full(const VerifyArgs& a, int dtype, bool aligned, bool draft_aligned, int grid,
+                               cudaStream_t s) {
+    const int64_t rows = (int64_t)a.n.B * (a.n.N + 1);
+    const dim3 gp((unsigned)((rows + kWarps - 1) / kWarps));
+    cudaError_t err = (dtype == 1) ? launch_dependent(verify_prep_kernel<1>, gp, dim3(kThreads), 0, s, a)
+                                   : launch_dependent(verify_prep_kernel<0>, gp, dim3(kThreads), 0, s, a);
+    if (err != cudaSuccess) return err;
+    auto go = [&](auto kern, dim3 g) { return launch_dependent(kern, g, dim3(kThreads), 0, s, a); };
+    if (dtype == 1) err = aligned ? go(verify_stream_kernel<1, true>, dim3(grid)) : go(verify_stream_kernel<1, false>, dim3(grid));
+    else err = aligned ? go(verify_stream_kernel<0, true>, dim3(grid)) : go(verify_stream_kernel<0, false>, dim3(grid));
+    if (err != cudaSuccess) return err;
+    const dim3 go_rows((unsigned)rows);
+    if (dtype == 1) {
+        if (aligned && draft_aligned) err = go(full_overlap_kernel<1, true, true>, go_rows);
+        else err = go(full_overlap_kernel<1, false, false>, go_rows);
+    } else {
+        if (aligned && draft_aligned) err = go(full_overlap_kernel<0, true, true>, go_rows);
+        else err = go(full_overlap_kernel<0, false, false>, go_rows);
+    }
+    if (err != cudaSuccess) return err;
+    const dim3 g2((a.n.V + kResChunk - 1) / kResChunk, a.n.B);
+    if (dtype == 1) {
+        if (aligned && draft_aligned) return go(residual_kernel<1, true, true, true>, g2);
+        return go(residual_kernel<1, false, true, false>, g2);
+    }
+    if (aligned && draft_aligned) return go(residual_kernel<0, true, true, true>, g2);
+    return go(residual_kernel<0, false, true, false>, g2);
 }
 
 cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid, cudaStream_t s) {

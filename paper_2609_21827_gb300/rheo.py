@@ -21,7 +21,7 @@ STATUS_BAD_LOGIT, STATUS_EMPTY_ROW, STATUS_BAD_TEMPERATURE, STATUS_INTERNAL = 1,
 SLOT_ROOT, SLOT_LEAD, SLOT_SAMPLED, SLOT_FILL = 0, 1, 2, 3
 
 EXPORTS = ("rheo_sizes", "rheo_workspace_init", "rheo_expand", "rheo_prune", "rheo_verify", "rheo_verify_static",
-           "rheo_tree_attention", "rheo_verify_variant",
+           "rheo_tree_attention", "rheo_verify_variant", "rheo_verify_full",
            "rheo_get_status")
 
 
@@ -86,6 +86,9 @@ def lib():
         L.rheo_verify_variant.argtypes = [C, ctypes.c_int32, _VP, ctypes.c_int64, _VP, _VP, _VP,
                                           ctypes.POINTER(_Tree), ctypes.POINTER(_Pruned), ctypes.POINTER(_VerifyOut),
                                           _VP, _VP]
+        L.rheo_verify_full.argtypes = [C, _VP, ctypes.c_int64, _VP, ctypes.c_int64, _VP, _VP, _VP,
+                                       ctypes.POINTER(_Tree), ctypes.POINTER(_Pruned), ctypes.POINTER(_VerifyOut),
+                                       _VP, _VP]
         L.rheo_tree_attention.argtypes = [C, ctypes.POINTER(_Pruned), ctypes.POINTER(_TreeAttn), _VP, _VP]
         for name in EXPORTS:
             getattr(L, name).restype = ctypes.c_int
@@ -286,6 +289,26 @@ def verify_variant(cfg: Config, variant: int, logits: torch.Tensor, temperature:
                                      ctypes.byref(tree.c()), ctypes.byref(pruned.c()), ctypes.byref(out.c()),
                                      ws.ptr(), _stream(stream)),
            "rheo_verify_variant")
+
+
+def verify_full(cfg: Config, logits: torch.Tensor, draft_rows: list, temperature: torch.Tensor, seed: torch.Tensor,
+                offset: torch.Tensor, tree: Tree, pruned: Pruned, out: VerifyOut, ws: Workspace, stream=None) -> None:
+    """rheo_verify_full: draft_rows[d-1] = the [B, F_d, V] rows given to expand at depth d."""
+    stride = _rows(cfg, logits, cfg.batch * (cfg.budget + 1))
+    dstride = None
+    ptrs = (ctypes.c_void_p * cfg.depth)()
+    for d, x in enumerate(draft_rows):
+        st = _rows(cfg, x, x.shape[0] * x.shape[1])
+        if dstride is None:
+            dstride = st
+        elif st != dstride:
+            raise RheoError("draft rows of every depth need the same row stride")
+        ptrs[d] = x.data_ptr()
+    _check(lib().rheo_verify_full(ctypes.byref(cfg.c()), logits.data_ptr(), stride, ptrs, dstride,
+                                  _f32(temperature).data_ptr(), _i64(seed).data_ptr(), _i64(offset).data_ptr(),
+                                  ctypes.byref(tree.c()), ctypes.byref(pruned.c()), ctypes.byref(out.c()), ws.ptr(),
+                                  _stream(stream)),
+           "rheo_verify_full")
 
 
 def verify_static(cfg: Config, logits: torch.Tensor, temperature: torch.Tensor, seed: torch.Tensor,

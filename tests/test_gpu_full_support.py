@@ -101,3 +101,64 @@ def test_full_support_requires_m_at_most_one():
 def test_full_support_tree_parity_qwen3_size():
     w = synth.WORKLOADS["qwen3_batch"]
     assert _run(w, [1, 12]) <= 1
+
+
+def _cycle(w, reqs):
+    """Full cycle with full support on both sides; returns (explained flips, requests compared)."""
+    import oracle
+    cfg = _cfg(w)
+    draft = synth.make_draft_inputs(w, device="cuda")
+    tree, pr, ws, out = rheo.Tree(cfg), rheo.Pruned(cfg), rheo.Workspace(cfg), rheo.VerifyOut(cfg)
+    frontiers = []
+    for d in range(1, cfg.depth + 1):
+        rheo.expand(cfg, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tree, ws)
+        if d < cfg.depth:
+            frontiers.append(tree.frontier.clone())
+    rheo.prune(cfg, tree, pr, ws)
+    tgt = synth.target_rows(w, draft, frontiers, pr.gen_id)
+    rheo.verify_full(cfg, tgt, draft.rows, draft.temperature, draft.seed, draft.offset, tree, pr, out, ws)
+    assert rheo.status(cfg, ws) == 0
+    ocfg = oracle.Config(B=len(reqs), V=w.vocab, K=w.K, m=w.m, S=0, D=w.depth, N=w.budget, eps=cfg.eps)
+    ot = oracle.Tree(ocfg)
+    T = draft.temperature.cpu().numpy()[reqs]
+    seed, off = ph.u64(draft.seed)[reqs], ph.u64(draft.offset)[reqs]
+    ofr = []
+    for d in range(1, w.depth + 1):
+        oracle.expand(ocfg, d, draft.rows[d - 1][reqs].float().cpu().numpy(), T, seed, off, ot)
+        if d < w.depth:
+            ofr.append(ot.frontier.copy())
+    op = oracle.prune(ocfg, ot)
+    sub = synth.DraftInputs(w, [r_[reqs] for r_ in draft.rows], draft.temperature[reqs], draft.seed[reqs],
+                            draft.offset[reqs])
+    otg = synth.target_rows(w, sub, [torch.from_numpy(f) for f in ofr], torch.from_numpy(op.gen_id.copy()),
+                            device=draft.rows[0].device, request_ids=reqs)
+    oo = oracle.verify(ocfg, otg.float().cpu().numpy(), T, seed, off, ot, op)
+    explained = 0
+    gl, gt, gb = out.accepted_len.cpu().numpy(), out.accepted_tokens.cpu().numpy(), out.bonus_token.cpu().numpy()
+    for j, b in enumerate(reqs):
+        same = (gl[b] == oo.accepted_len[j] and np.array_equal(gt[b], oo.accepted_tokens[j])
+                and gb[b] == oo.bonus_token[j])
+        if not same:
+            gap = min(float(np.min(ot.gap_sample[j])), float(np.min(ot.gap_frontier[j])), float(op.gap_prune[j]),
+                      float(np.min(oo.gap_level[j])))
+            assert gap < ph.GAP, f"{w.name} request {b}: verification differs, oracle margin {gap}"
+            explained += 1
+    return explained
+
+
+@pytest.mark.parametrize("w", CASES, ids=[w.name for w in CASES])
+def test_full_support_verification_parity(w):
+    assert _cycle(w, list(range(w.batch))) <= 1
+
+
+def test_full_support_verification_parity_qwen3_size():
+    w = synth.WORKLOADS["qwen3_batch"]
+    assert _cycle(w, [4, 13]) <= 1
+
+
+def test_sparse_entry_points_reject_full_support():
+    import ctypes
+    cfg = _cfg(CASES[0])
+    rc = rheo.lib().rheo_verify_variant(ctypes.byref(cfg.c()), 0, None, 0, None, None, None, None, None, None,
+                                        None, None)
+    assert rc == rheo.RHEO_EINVAL

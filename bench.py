@@ -271,6 +271,9 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (a smaller case of the same kernels, for profiling)")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the verification variants, the synthetic-model cycles and the full-support step "
+                         "(for launch lists of the tree step alone)")
     ap.add_argument("--depth", type=int, default=0,
                     help="override the workload's depth (fewer expansion launches of the same shape, for profiling)")
     args = ap.parse_args(argv)
@@ -384,140 +387,142 @@ def main(argv=None):
     ver_ms /= n_k
     assert rheo.status(cfg, ws, stream) == 0
 
-    # tree-attention inputs of the target forward (not part of the tree step):
-    # 20 launches in one graph, averaged over replays
-    attn = rheo.TreeAttn(cfg, device=device)
-    g_attn = torch.cuda.CUDAGraph()
-    with torch.cuda.stream(stream):
-        rheo.tree_attention(cfg, pr, attn, ws, stream)
-        stream.synchronize()
-        with torch.cuda.graph(g_attn, stream=stream):
-            for _ in range(20):
-                rheo.tree_attention(cfg, pr, attn, ws, stream)
-        for _ in range(3):
-            g_attn.replay()
-        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a0.record(stream)
-        for _ in range(10):
-            g_attn.replay()
-        a1.record(stream)
-        stream.synchronize()
-    attn_us = a0.elapsed_time(a1) * 1e3 / 200
-    assert rheo.status(cfg, ws, stream) == 0
 
-    # verification variants (App. A, App. D.2) on the same trees and targets:
-    # per-call time on this step's tree, and the mean accepted length over the
-    # requests of 8 more cycles (Philox offsets 1..8), paired across variants
-    variants = {}
-    names = {"rheo": rheo.VERIFY_RHEO, "rrsw": rheo.VERIFY_RRSW, "onehot": rheo.VERIFY_ONEHOT}
-    vout = rheo.VerifyOut(cfg, row_lse=False, device=device)
-    for name, v in names.items():
+    variants, synthetic_lm, full_support, attn_us = None, None, None, None
+    if not args.no_extras:
+        # tree-attention inputs of the target forward (not part of the tree step):
+        # 20 launches in one graph, averaged over replays
+        attn = rheo.TreeAttn(cfg, device=device)
+        g_attn = torch.cuda.CUDAGraph()
         with torch.cuda.stream(stream):
-            for _ in range(3):
-                rheo.verify_variant(cfg, v, target, draft.temperature, draft.seed, draft.offset, tree, pr, vout, ws,
-                                    stream)
-            v0, v1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            v0.record(stream)
-            for _ in range(50):
-                rheo.verify_variant(cfg, v, target, draft.temperature, draft.seed, draft.offset, tree, pr, vout, ws,
-                                    stream)
-            v1.record(stream)
+            rheo.tree_attention(cfg, pr, attn, ws, stream)
             stream.synchronize()
-        variants[name] = {"verify_us": v0.elapsed_time(v1) * 1e3 / 50, "accepted": []}
-    off0 = draft.offset.clone()
-    for off in range(1, 9):
-        draft.offset.fill_(off)
-        tr2, pr2 = rheo.Tree(cfg, device=device), rheo.Pruned(cfg, device=device)
-        fr2 = []
-        for d in range(1, D + 1):
-            rheo.expand(cfg, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tr2, ws)
-            if d < D:
-                fr2.append(tr2.frontier.clone())
-        rheo.prune(cfg, tr2, pr2, ws)
-        tg2 = synth.target_rows(w, draft, fr2, pr2.gen_id)
+            with torch.cuda.graph(g_attn, stream=stream):
+                for _ in range(20):
+                    rheo.tree_attention(cfg, pr, attn, ws, stream)
+            for _ in range(3):
+                g_attn.replay()
+            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a0.record(stream)
+            for _ in range(10):
+                g_attn.replay()
+            a1.record(stream)
+            stream.synchronize()
+        attn_us = a0.elapsed_time(a1) * 1e3 / 200
+        assert rheo.status(cfg, ws, stream) == 0
+        # verification variants (App. A, App. D.2) on the same trees and targets:
+        # per-call time on this step's tree, and the mean accepted length over the
+        # requests of 8 more cycles (Philox offsets 1..8), paired across variants
+        variants = {}
+        names = {"rheo": rheo.VERIFY_RHEO, "rrsw": rheo.VERIFY_RRSW, "onehot": rheo.VERIFY_ONEHOT}
+        vout = rheo.VerifyOut(cfg, row_lse=False, device=device)
         for name, v in names.items():
-            rheo.verify_variant(cfg, v, tg2, draft.temperature, draft.seed, draft.offset, tr2, pr2, vout, ws)
-            variants[name]["accepted"] += vout.accepted_len.cpu().tolist()
-    draft.offset.copy_(off0)
-    assert rheo.status(cfg, ws) == 0
-    for name in names:
-        acc = variants[name].pop("accepted")
-        variants[name]["mean_accepted"] = sum(acc) / len(acc)
-        variants[name]["samples"] = len(acc)
+            with torch.cuda.stream(stream):
+                for _ in range(3):
+                    rheo.verify_variant(cfg, v, target, draft.temperature, draft.seed, draft.offset, tree, pr, vout, ws,
+                                        stream)
+                v0, v1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                v0.record(stream)
+                for _ in range(50):
+                    rheo.verify_variant(cfg, v, target, draft.temperature, draft.seed, draft.offset, tree, pr, vout, ws,
+                                        stream)
+                v1.record(stream)
+                stream.synchronize()
+            variants[name] = {"verify_us": v0.elapsed_time(v1) * 1e3 / 50, "accepted": []}
+        off0 = draft.offset.clone()
+        for off in range(1, 9):
+            draft.offset.fill_(off)
+            tr2, pr2 = rheo.Tree(cfg, device=device), rheo.Pruned(cfg, device=device)
+            fr2 = []
+            for d in range(1, D + 1):
+                rheo.expand(cfg, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tr2, ws)
+                if d < D:
+                    fr2.append(tr2.frontier.clone())
+            rheo.prune(cfg, tr2, pr2, ws)
+            tg2 = synth.target_rows(w, draft, fr2, pr2.gen_id)
+            for name, v in names.items():
+                rheo.verify_variant(cfg, v, tg2, draft.temperature, draft.seed, draft.offset, tr2, pr2, vout, ws)
+                variants[name]["accepted"] += vout.accepted_len.cpu().tolist()
+        draft.offset.copy_(off0)
+        assert rheo.status(cfg, ws) == 0
+        for name in names:
+            acc = variants[name].pop("accepted")
+            variants[name]["mean_accepted"] = sum(acc) / len(acc)
+            variants[name]["samples"] = len(acc)
 
-    # synthetic analogue of the ablations over m and T (Sec. 5.3, Sec. 5.4):
-    # multi-cycle decoding against k-gram draft / target models (V = 64, k = 2),
-    # tau = mean tokens emitted per cycle
-    from paper_2609_21827_gb300 import cycles as cyc
-    lm_gen = torch.Generator().manual_seed(2609)
-    d_lm = cyc.KGramLM.random(64, 2, 1.5, lm_gen, device=device)
-    t_lm = cyc.KGramLM.random(64, 2, 1.5, lm_gen, device=device, base=d_lm, noise=0.8)
-    tau = {}
-    lm_ms = 0.0
-    for m_ in (0, 1, 2, 3):
-        for T_ in (0.5, 1.0):
-            c2 = rheo.Config(batch=1024, vocab=64, K=8, depth=6, budget=40, m=m_, support=64, dtype="f32")
-            win = torch.randint(0, 64, (1024, 2), generator=lm_gen).to(device)
-            sd = torch.arange(1024, dtype=torch.int64, device=device) * 7919 + 31 * m_ + int(10 * T_)
-            t0 = time.time()
-            res = cyc.run_cycles(c2, d_lm, t_lm, win, torch.full((1024,), T_), sd, cycles=6, L=1)
-            torch.cuda.synchronize()
-            lm_ms += (time.time() - t0) * 1e3 / 6
-            tau[f"m{m_}_T{T_}"] = float(res.accepted.float().mean().item()) + 1.0
-    synthetic_lm = {"vocab": 64, "k": 2, "K": 8, "depth": 6, "budget": 40, "sequences": 1024, "cycles": 6,
-                    "tau": tau, "host_ms_per_cycle": lm_ms / 8}
+        # synthetic analogue of the ablations over m and T (Sec. 5.3, Sec. 5.4):
+        # multi-cycle decoding against k-gram draft / target models (V = 64, k = 2),
+        # tau = mean tokens emitted per cycle
+        from paper_2609_21827_gb300 import cycles as cyc
+        lm_gen = torch.Generator().manual_seed(2609)
+        d_lm = cyc.KGramLM.random(64, 2, 1.5, lm_gen, device=device)
+        t_lm = cyc.KGramLM.random(64, 2, 1.5, lm_gen, device=device, base=d_lm, noise=0.8)
+        tau = {}
+        lm_ms = 0.0
+        for m_ in (0, 1, 2, 3):
+            for T_ in (0.5, 1.0):
+                c2 = rheo.Config(batch=1024, vocab=64, K=8, depth=6, budget=40, m=m_, support=64, dtype="f32")
+                win = torch.randint(0, 64, (1024, 2), generator=lm_gen).to(device)
+                sd = torch.arange(1024, dtype=torch.int64, device=device) * 7919 + 31 * m_ + int(10 * T_)
+                t0 = time.time()
+                res = cyc.run_cycles(c2, d_lm, t_lm, win, torch.full((1024,), T_), sd, cycles=6, L=1)
+                torch.cuda.synchronize()
+                lm_ms += (time.time() - t0) * 1e3 / 6
+                tau[f"m{m_}_T{T_}"] = float(res.accepted.float().mean().item()) + 1.0
+        synthetic_lm = {"vocab": 64, "k": 2, "K": 8, "depth": 6, "budget": 40, "sequences": 1024, "cycles": 6,
+                        "tau": tau, "host_ms_per_cycle": lm_ms / 8}
 
-    # full support (App. B, Table tab:sparse_support, row Full): the same
-    # workload with the sampled token drawn over the whole vocabulary; a graph
-    # of its 12 launches timed like the main step, plus per-call times
-    cfg_f = rheo.Config(batch=w.batch, vocab=w.vocab, K=w.K, depth=w.depth, budget=w.budget, m=w.m, support=0,
-                        dtype=w.dtype)
-    tf, pf, wf = rheo.Tree(cfg_f, device), rheo.Pruned(cfg_f, device), rheo.Workspace(cfg_f, device)
-    of = rheo.VerifyOut(cfg_f, row_lse=False, device=device)
-    fr_f = []
-    for d in range(1, D + 1):
-        rheo.expand(cfg_f, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tf, wf)
-        if d < D:
-            fr_f.append(tf.frontier.clone())
-    rheo.prune(cfg_f, tf, pf, wf)
-    tgt_f = synth.target_rows(w, draft, fr_f, pf.gen_id)
-
-    def step_f(s_, marks=None):
+        # full support (App. B, Table tab:sparse_support, row Full): the same
+        # workload with the sampled token drawn over the whole vocabulary; a graph
+        # of its 12 launches timed like the main step, plus per-call times
+        cfg_f = rheo.Config(batch=w.batch, vocab=w.vocab, K=w.K, depth=w.depth, budget=w.budget, m=w.m, support=0,
+                            dtype=w.dtype)
+        tf, pf, wf = rheo.Tree(cfg_f, device), rheo.Pruned(cfg_f, device), rheo.Workspace(cfg_f, device)
+        of = rheo.VerifyOut(cfg_f, row_lse=False, device=device)
+        fr_f = []
         for d in range(1, D + 1):
-            rheo.expand(cfg_f, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tf, wf, s_)
-        if marks:
-            marks[0].record(s_)
-        rheo.prune(cfg_f, tf, pf, wf, s_)
-        if marks:
-            marks[1].record(s_)
-        rheo.verify_full(cfg_f, tgt_f, draft.rows, draft.temperature, draft.seed, draft.offset, tf, pf, of, wf, s_)
+            rheo.expand(cfg_f, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tf, wf)
+            if d < D:
+                fr_f.append(tf.frontier.clone())
+        rheo.prune(cfg_f, tf, pf, wf)
+        tgt_f = synth.target_rows(w, draft, fr_f, pf.gen_id)
 
-    g_f = torch.cuda.CUDAGraph()
-    with torch.cuda.stream(stream):
-        step_f(stream)
-        stream.synchronize()
-        with torch.cuda.graph(g_f, stream=stream):
+        def step_f(s_, marks=None):
+            for d in range(1, D + 1):
+                rheo.expand(cfg_f, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tf, wf, s_)
+            if marks:
+                marks[0].record(s_)
+            rheo.prune(cfg_f, tf, pf, wf, s_)
+            if marks:
+                marks[1].record(s_)
+            rheo.verify_full(cfg_f, tgt_f, draft.rows, draft.temperature, draft.seed, draft.offset, tf, pf, of, wf, s_)
+
+        g_f = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(stream):
             step_f(stream)
-        for _ in range(3):
-            g_f.replay()
-        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        n_f = max(20, min(200, args.steps))
-        f0.record(stream)
-        for _ in range(n_f):
-            g_f.replay()
-        f1.record(stream)
-        stream.synchronize()
-        ms_f = f0.elapsed_time(f1) / n_f
-        mk = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
-        mk[0].record(stream)
-        step_f(stream, marks=(mk[1], mk[2]))
-        mk[3].record(stream)
-        stream.synchronize()
-    assert rheo.status(cfg_f, wf, stream) == 0
-    full_support = {"tree_steps_per_s": 1e3 / ms_f, "ms_per_step": ms_f,
-                    "expand_ms": mk[0].elapsed_time(mk[1]), "prune_ms": mk[1].elapsed_time(mk[2]),
-                    "verify_ms": mk[2].elapsed_time(mk[3]),
-                    "note": "eager per-call times; the step time is the CUDA graph of its 12 launches"}
+            stream.synchronize()
+            with torch.cuda.graph(g_f, stream=stream):
+                step_f(stream)
+            for _ in range(3):
+                g_f.replay()
+            f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            n_f = max(20, min(200, args.steps))
+            f0.record(stream)
+            for _ in range(n_f):
+                g_f.replay()
+            f1.record(stream)
+            stream.synchronize()
+            ms_f = f0.elapsed_time(f1) / n_f
+            mk = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+            mk[0].record(stream)
+            step_f(stream, marks=(mk[1], mk[2]))
+            mk[3].record(stream)
+            stream.synchronize()
+        assert rheo.status(cfg_f, wf, stream) == 0
+        full_support = {"tree_steps_per_s": 1e3 / ms_f, "ms_per_step": ms_f,
+                        "expand_ms": mk[0].elapsed_time(mk[1]), "prune_ms": mk[1].elapsed_time(mk[2]),
+                        "verify_ms": mk[2].elapsed_time(mk[3]),
+                        "note": "eager per-call times; the step time is the CUDA graph of its 12 launches"}
 
     # end to end through the public API with host buffers: H2D of every input, D2H of the results
     e2e = None

@@ -82,6 +82,7 @@ constexpr int kMaxFullDepth = 32;  // depth limit of full-support verification
 struct VerifyArgs {
     Dims n;                         // n.chunks: 2 KB chunks per target row
     int variant = kVerifyRheo;      // verification rule at every node (kVerify*)
+    int prep_grid = 0;              // CTAs of the prep launch (0: one per two rows)
     int units;                      // warps of the stream launch with work (one contiguous run of chunks each)
     const char* logits;
     int64_t row_stride_bytes;

@@ -120,17 +120,18 @@ __device__ __forceinline__ void load_chunk(uint4 (&v)[kCV], const char* row, int
 //   cx, tx     l / T as float-float at the children and at the tail tokens
 //   coin       the node's K+2 Philox coins
 constexpr int kHdr = 8;
+// prep runs beside the stream launch: two stream CTAs per SM capped at 96
+// registers a thread leave room for one prep CTA of 256 threads
+constexpr int kPrepThreads = 256;
+constexpr int kStreamMaxRegs = 96;
 
 // One warp per pruned row: the row's record.
 template <int DT>
-__global__ void __launch_bounds__(kThreads) verify_prep_kernel(const VerifyArgs a) {
+__device__ void prep_row(const VerifyArgs& a, int64_t r) {
     using E = Elem<DT>;
-    grid_dependency_begin();
     const Dims& n = a.n;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
     const int K = n.K, TL = n.TL, NP = n.N + 1, m = n.m;
-    const int64_t r = (int64_t)blockIdx.x * kWarps + warp;
-    if (r >= (int64_t)n.B * NP) return;
     const int b = (int)(r / NP);
     const int64_t pb = (int64_t)b * NP, nb = (int64_t)b * n.G1;
     int nc = a.pr.n_child[r], fc = a.pr.first_child[r], sc = a.pr.sampled_child[r];
@@ -221,6 +222,19 @@ __global__ void __launch_bounds__(kThreads) verify_prep_kernel(const VerifyArgs 
         hdr[3] = gen;
         hdr[4] = __float_as_int(qs);
     }
+}
+
+// One warp per pruned row (the grid may be capped, each warp then taking rows in
+// turn); it runs beside the stream launch and must end before the stream
+// launch's first row finalises, so it keeps one row per warp.
+template <int DT>
+__global__ void __launch_bounds__(kPrepThreads) verify_prep_kernel(const VerifyArgs a) {
+    grid_dependency_begin();
+    const int64_t rows = (int64_t)a.n.B * (a.n.N + 1);
+    const int w = threadIdx.x >> 5;
+    for (int64_t r = (int64_t)blockIdx.x * (kPrepThreads / 32) + w; r < rows;
+         r += (int64_t)gridDim.x * (kPrepThreads / 32))
+        prep_row<DT>(a, r);
 }
 
 // exp(x - c) for x = l / T and c as float-float (the arithmetic of exp_scaled_minus)
@@ -449,7 +463,7 @@ __device__ __noinline__ void finalize_row(const VerifyArgs& a, int64_t r, WarpRo
 }
 
 template <int DT, bool ALIGNED>
-__global__ void __launch_bounds__(kThreads, 2) verify_stream_kernel(const VerifyArgs a) {
+__global__ void __maxnreg__(kStreamMaxRegs) verify_stream_kernel(const VerifyArgs a) {
     // streaming needs nothing from the grids before this one: let the next grid
     // launch now, and wait for the row records only before the first table
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -631,6 +645,17 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
         lead = (n.m == 1) ? a.tree.token[(int64_t)b * n.G1 + gs - 1] : -1;
     }
 
+    // this thread's elements of the stopping row (and, with full support after
+    // a rejection, of its draft row), requested before the candidates' records
+    // so that both round trips overlap
+    const int64_t e0 = e_lo + (int64_t)tid * kResPer;
+    uint4 xv[kResPer / E::VEC];
+    uint4 dv[kResPer / E::VEC];
+#pragma unroll
+    for (int j = 0; j < kResPer / E::VEC; ++j) {
+        xv[j] = load_vec<DT, ALIGNED>(row, e0 + j * E::VEC, V);
+        if (FULL && drow) dv[j] = load_vec<DT, DALIGNED>(drow, e0 + j * E::VEC, V);
+    }
     for (int c = tid; c < nc_ok; c += kThreads) {
         const int tok = __ldcg(rchild + 3 * c);
         if (tok >= e_lo && tok < e_lo + kResChunk)
@@ -648,14 +673,6 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     // elsewhere, over V minus the candidates
     unsigned long long best = 0ull;
     {
-        const int64_t e0 = e_lo + (int64_t)tid * kResPer;
-        uint4 xv[kResPer / E::VEC];  // this thread's elements of the stopping row
-        uint4 dv[kResPer / E::VEC];  // full support: the same elements of the draft row
-#pragma unroll
-        for (int j = 0; j < kResPer / E::VEC; ++j) {
-            xv[j] = load_vec<DT, ALIGNED>(row, e0 + j * E::VEC, V);
-            if (FULL && drow) dv[j] = load_vec<DT, DALIGNED>(drow, e0 + j * E::VEC, V);
-        }
 #pragma unroll
         for (int h = 0; h < kResPer / 4; ++h) {
             if (e0 + 4 * h >= V) break;
@@ -832,9 +849,10 @@ __global__ void __launch_bounds__(kThreads) full_overlap_kernel(const VerifyArgs
 cudaError_t launch_verify_full(const VerifyArgs& a, int dtype, bool aligned, bool draft_aligned, int grid,
                                cudaStream_t s) {
     const int64_t rows = (int64_t)a.n.B * (a.n.N + 1);
-    const dim3 gp((unsigned)((rows + kWarps - 1) / kWarps));
-    cudaError_t err = (dtype == 1) ? launch_dependent(verify_prep_kernel<1>, gp, dim3(kThreads), 0, s, a)
-                                   : launch_dependent(verify_prep_kernel<0>, gp, dim3(kThreads), 0, s, a);
+    const int64_t prep_ctas = (rows + kPrepThreads / 32 - 1) / (kPrepThreads / 32);
+    const dim3 gp((unsigned)(a.prep_grid > 0 && a.prep_grid < prep_ctas ? a.prep_grid : prep_ctas));
+    cudaError_t err = (dtype == 1) ? launch_dependent(verify_prep_kernel<1>, gp, dim3(kPrepThreads), 0, s, a)
+                                   : launch_dependent(verify_prep_kernel<0>, gp, dim3(kPrepThreads), 0, s, a);
     if (err != cudaSuccess) return err;
     auto go = [&](auto kern, dim3 g) { return launch_dependent(kern, g, dim3(kThreads), 0, s, a); };
     if (dtype == 1) err = aligned ? go(verify_stream_kernel<1, true>, dim3(grid)) : go(verify_stream_kernel<1, false>, dim3(grid));
@@ -860,9 +878,10 @@ cudaError_t launch_verify_full(const VerifyArgs& a, int dtype, bool aligned, boo
 
 cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid, cudaStream_t s) {
     const int64_t rows = (int64_t)a.n.B * (a.n.N + 1);
-    const dim3 gp((unsigned)((rows + kWarps - 1) / kWarps));
-    cudaError_t e0 = (dtype == 1) ? launch_dependent(verify_prep_kernel<1>, gp, dim3(kThreads), 0, s, a)
-                                  : launch_dependent(verify_prep_kernel<0>, gp, dim3(kThreads), 0, s, a);
+    const int64_t prep_ctas = (rows + kPrepThreads / 32 - 1) / (kPrepThreads / 32);
+    const dim3 gp((unsigned)(a.prep_grid > 0 && a.prep_grid < prep_ctas ? a.prep_grid : prep_ctas));
+    cudaError_t e0 = (dtype == 1) ? launch_dependent(verify_prep_kernel<1>, gp, dim3(kPrepThreads), 0, s, a)
+                                  : launch_dependent(verify_prep_kernel<0>, gp, dim3(kPrepThreads), 0, s, a);
     if (e0 != cudaSuccess) return e0;
     auto go_stream = [&](auto kern) {
         return launch_dependent(kern, dim3(grid), dim3(kThreads), 0, s, a);

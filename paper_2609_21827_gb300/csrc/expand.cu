@@ -819,17 +819,14 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             if (tid == 0) e2.bad = (got != S) ? 1 : 0;
         }
         __syncthreads();
-
-        __syncthreads();
         const float lse1 = e2.lse1;
-        if (tid < S) {
+        if (tid < S) {  // read by others only after the next barrier
             const unsigned long long x = e2.sorted[tid];
             e2.id[tid] = (int32_t)(0xFFFFFFFFu - (uint32_t)x);
             const float l = E::value_of_key((uint32_t)(x >> 32));
             e2.l[tid] = l;
             e2.lq0[tid] = __fsub_rn(l, lse1);
         }
-        __syncthreads();
 
         const float T = s_pre.T;
         const uint64_t seed = s_pre.seed, off = s_pre.off;
@@ -843,19 +840,23 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
         const int64_t g0 = depth_base(K, a.d) + (int64_t)f * (K + 1);
 
         if constexpr (!FULL) {
-            // tempered tail q~ = softmax(l / T) over support ranks m+1..S; Y by Gumbel-max
-            const float tau = (tid < TL) ? __fdiv_rn(e2.l[m + tid], T) : -INFINITY;
-            const float mt = __fdiv_rn(e2.l[m], T);  // the support is sorted: rank m is the tail's maximum
-            const FF st = red_sum_ff<kXWarps>(FF{(tid < TL && mt > -INFINITY) ? expf(tau - mt) : 0.0f, 0.0f}, red, par);
-            const FF lse_tail = ff_add(ff_log(st), mt);
+            // tempered tail q~ = softmax(l / T) over support ranks m+1..S; Y by
+            // Gumbel-max (the key needs no partition sum: one reduction for both)
+            auto lof = [&](int i) { return E::value_of_key((uint32_t)(e2.sorted[i] >> 32)); };
+            const float tau = (tid < TL) ? __fdiv_rn(lof(m + tid), T) : -INFINITY;
+            const float mt = __fdiv_rn(lof(m), T);  // the support is sorted: rank m is the tail's maximum
             unsigned long long pack = 0ull;
             if (tid < TL) {
-                e2.q[tid] = expf(__fsub_rn(tau, lse_tail.hi) - lse_tail.lo);
                 const float g = gumbel(uniform(seed, off, kTagSample, (int)par_g, (uint64_t)tid));
                 const float key = __fadd_rn(tau, g);
                 if (key > -INFINITY) pack = make_key(ord_f32(key), tid);
             }
-            const unsigned long long bestp = red_max_u64<kXWarps>(pack, red, par);
+            FF st;
+            unsigned long long bestp;
+            red_sum_ff_max_u64<kXWarps>(FF{(tid < TL && mt > -INFINITY) ? expf(tau - mt) : 0.0f, 0.0f}, pack, red, par,
+                                        st, bestp);
+            const FF lse_tail = ff_add(ff_log(st), mt);
+            if (tid < TL) e2.q[tid] = expf(__fsub_rn(tau, lse_tail.hi) - lse_tail.lo);
             if (tid == 0) {
                 e2.best = bestp ? (int)(0xFFFFFFFFu - (uint32_t)bestp) : 0;
                 e2.lse_tail = __fadd_rn(lse_tail.hi, lse_tail.lo);
@@ -868,7 +869,8 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             float MT;
             const float mT = __fdiv_rn(mu, fT);
             float sT = f2_fold(sumT2);
-            if (m == 1 && kid >= 0 && kid != e2.id[0])  // kept out, and not the lead: it belongs to the tail
+            const int lead_id = (int)(0xFFFFFFFFu - (uint32_t)e2.sorted[0]);  // e2.id is not published yet
+            if (m == 1 && kid >= 0 && kid != lead_id)  // kept out, and not the lead: it belongs to the tail
                 sT += fast_exp2(fmaf(__fdiv_rn(kx, fT), kLog2e, -mT * kLog2e));
             const FF ST = red_partition<kXWarps>(mT, sT, kLog2e, MT, red, par);  // the tail's sum
             for (int q = 0; q <= m; ++q) {
@@ -974,6 +976,10 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             a.tree.qtilde[g] = qv;
             a.tree.slot[g] = st8;
         }
+        // ---- last row of the request: the K best depth-d nodes become the frontier ----
+        // (the arrival waits only for the children's writes: the tail lists, read
+        // by no one before verification, are written after it)
+        const bool last_row = arrive_last(a.req_ticket + b, (unsigned)a.F, bs);
         if (tid < TL) {
             const int64_t q0 = ((int64_t)b * n.E + eidx) * TL;
             a.tree.tail_ids[q0 + tid] = e2.id[m + tid];
@@ -983,9 +989,7 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             a.tree.lse1[(int64_t)b * n.E + eidx] = lse1;
             if (a.tree.lse_tail) a.tree.lse_tail[(int64_t)b * n.E + eidx] = e2.lse_tail;
         }
-
-        // ---- last row of the request: the K best depth-d nodes become the frontier ----
-        if (!arrive_last(a.req_ticket + b, (unsigned)a.F, bs)) return;
+        if (!last_row) return;
         if (a.d == n.D) return;
         {
             const int nn = a.F * (K + 1);

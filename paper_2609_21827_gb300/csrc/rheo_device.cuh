@@ -492,6 +492,41 @@ __device__ __forceinline__ FF red_sum_ff(FF v, Red& r, int& par) {
     return FF{__shfl_sync(0xFFFFFFFFu, t.hi, 0), __shfl_sync(0xFFFFFFFFu, t.lo, 0)};
 }
 
+// Block sum (float-float) and maximum (u64) in one barrier: both partials of
+// every warp go to the scratch at once, then the same shuffle trees as
+// red_sum_ff and red_max_u64 combine them in every warp.
+template <int NW = kWarps>
+__device__ __forceinline__ void red_sum_ff_max_u64(FF v, unsigned long long k, Red& r, int& par, FF& sum,
+                                                   unsigned long long& mx) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        v = ff_add(v, ff_shfl_xor(v, o));
+        const unsigned long long y = __shfl_xor_sync(0xFFFFFFFFu, k, o);
+        k = y > k ? y : k;
+    }
+    float* bh = r.f[par];
+    float* bl = r.g[par];
+    unsigned long long* bu = r.u[par];
+    par ^= 1;
+    if ((threadIdx.x & 31) == 0) {
+        bh[threadIdx.x >> 5] = v.hi;
+        bl[threadIdx.x >> 5] = v.lo;
+        bu[threadIdx.x >> 5] = k;
+    }
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    FF t = lane < NW ? FF{bh[lane], bl[lane]} : FF{0.0f, 0.0f};
+    unsigned long long q = lane < NW ? bu[lane] : 0ull;
+#pragma unroll
+    for (int o = NW / 2; o > 0; o >>= 1) {
+        t = ff_add(t, ff_shfl_xor(t, o));
+        const unsigned long long y = __shfl_xor_sync(0xFFFFFFFFu, q, o);
+        q = y > q ? y : q;
+    }
+    sum = FF{__shfl_sync(0xFFFFFFFFu, t.hi, 0), __shfl_sync(0xFFFFFFFFu, t.lo, 0)};
+    mx = __shfl_sync(0xFFFFFFFFu, q, 0);
+}
+
 template <int NW = kWarps>
 __device__ __forceinline__ unsigned long long red_max_u64(unsigned long long v, Red& r, int& par) {
     v = warp_max_u64(v);

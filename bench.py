@@ -541,19 +541,45 @@ def main(argv=None):
             sum(x.numel() * x.element_size() for x in (h_T, h_seed, h_off))
         d2h = sum(x.numel() * x.element_size() for x in res)
 
+        # the inputs are copied on two copy streams while the kernels run: the
+        # rows of depth d (and the target rows) on their own, each kernel waiting
+        # only for the copies it reads, each copy waiting only for the previous
+        # step's kernel that reads the same buffer
+        cstreams = [torch.cuda.Stream(device=device), torch.cuda.Stream(device=device)]
+        ev_rows = [torch.cuda.Event() for _ in range(D)]
+        ev_rows_used = [torch.cuda.Event() for _ in range(D)]
+        ev_small, ev_tgt, ev_step = torch.cuda.Event(), torch.cuda.Event(), torch.cuda.Event()
+        ev_step.record(stream)
+
         def e2e_step(s):
-            for hr, dr in zip(h_rows, d_rows):
-                dr.copy_(hr, non_blocking=True)
-            d_tgt.copy_(h_tgt, non_blocking=True)
-            d_T.copy_(h_T, non_blocking=True)
-            d_seed.copy_(h_seed, non_blocking=True)
-            d_off.copy_(h_off, non_blocking=True)
+            c0, c1 = cstreams
+            c0.wait_event(ev_step)  # the small inputs are read by every kernel of the step
+            with torch.cuda.stream(c0):
+                d_T.copy_(h_T, non_blocking=True)
+                d_seed.copy_(h_seed, non_blocking=True)
+                d_off.copy_(h_off, non_blocking=True)
+                ev_small.record(c0)
+            for d in range(D):
+                cs = cstreams[d % 2]
+                cs.wait_event(ev_rows_used[d])
+                with torch.cuda.stream(cs):
+                    d_rows[d].copy_(h_rows[d], non_blocking=True)
+                    ev_rows[d].record(cs)
+            c1.wait_event(ev_step)
+            with torch.cuda.stream(c1):
+                d_tgt.copy_(h_tgt, non_blocking=True)
+                ev_tgt.record(c1)
+            s.wait_event(ev_small)
             for d in range(1, D + 1):
+                s.wait_event(ev_rows[d - 1])
                 rheo.expand(cfg, d, d_rows[d - 1], d_T, d_seed, d_off, tree, ws, s)
+                ev_rows_used[d - 1].record(s)
             rheo.prune(cfg, tree, pr, ws, s)
+            s.wait_event(ev_tgt)
             rheo.verify(cfg, d_tgt, d_T, d_seed, d_off, tree, pr, out, ws, s)
             for x, h in zip((out.accepted_len, out.accepted_tokens, out.bonus_token), res):
                 h.copy_(x, non_blocking=True)
+            ev_step.record(s)
 
         with torch.cuda.stream(stream):
             for _ in range(3):
@@ -566,6 +592,7 @@ def main(argv=None):
                 e2e_step(stream)
             e1.record(stream)
             stream.synchronize()
+            torch.cuda.synchronize()
         e2e_s = reduce_max_time(e0.elapsed_time(e1) / 1e3, world, device)
         e2e = {"value": world * args.e2e_steps / e2e_s, "unit": "tree-steps/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h}

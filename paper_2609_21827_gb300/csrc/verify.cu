@@ -556,6 +556,7 @@ constexpr int kStageRows = 1024; // pruned rows whose verdicts the walk stages i
 __device__ __forceinline__ unsigned long long pack_key(float key, int64_t id) {
     return ((unsigned long long)ord_f32(key) << 32) | (0xFFFFFFFFu - (uint32_t)id);
 }
+__device__ __forceinline__ float key_of_pack(unsigned long long pk) { return Elem<0>::value_of_key((uint32_t)(pk >> 32)); }
 
 // Full support (FULL): every token but the lead belongs to the tail, so after a
 // rejection the key of each token outside the candidates is log r^ + g with
@@ -672,7 +673,7 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     // key of the draw from r: log r^ + g on the tail (after a rejection), log p + g
     // elsewhere, over V minus the candidates
     unsigned long long best = 0ull;
-    {
+    if (FULL && drow) {
 #pragma unroll
         for (int h = 0; h < kResPer / 4; ++h) {
             if (e0 + 4 * h >= V) break;
@@ -687,7 +688,7 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
                 const float x = E::value(E::raw(xv[q / E::VEC], q % E::VEC));
                 const float g = gumbel(u01(word_of(rnd, i)));
                 float key;
-                if (FULL && drow && id != lead) {
+                if (id != lead) {
                     const float pt = exp_ff_minus(ff_div(x, T), lse_ff);
                     const float xd = E::value(E::raw(dv[q / E::VEC], q % E::VEC));
                     const float qt = expf(__fsub_rn(__fdiv_rn(xd, T), lt.hi) - lt.lo);
@@ -699,6 +700,62 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
                 }
                 if (key > -INFINITY) {
                     const unsigned long long pk = pack_key(key, id);
+                    best = pk > best ? pk : best;
+                }
+            }
+        }
+    } else {
+        // key = fp32(lp + g), lp = fp32(l/T - lse).  Exact filter: the warp's best
+        // key among each thread's highest-lp token is a lower bound B0 of the
+        // winning key; g never exceeds kGumbelMax, so a token with lp + kGumbelMax
+        // < B0 cannot win (no uniform drawn); otherwise it can beat B0 only if
+        // u > exp(-exp(lp - B0)), tested with a 1e-4 margin; the rest get the
+        // exact key.
+        constexpr float kGumbelMax = 16.7f;  // -log(-log u) at the largest uniform is 16.636
+        float lp[kResPer];
+        int top = -1;
+#pragma unroll
+        for (int q = 0; q < kResPer; ++q) {
+            const int64_t id = e0 + q;
+            const int li = (int)(id - e_lo);
+            const bool ok = id < V && !(((excl_bits[li >> 5] | tail_bits[li >> 5]) >> (li & 31)) & 1u);
+            lp[q] = ok ? __fsub_rn(__fdiv_rn(E::value(E::raw(xv[q / E::VEC], q % E::VEC)), T), lse) : -INFINITY;
+            if (lp[q] > -INFINITY && (top < 0 || lp[q] > lp[top])) top = q;
+        }
+        auto exact_key = [&](int q) {
+            const float u = u01(word_of(philox_block(seed, off, kTagResidual, gen_u, (uint64_t)((e0 + q) >> 2)),
+                                        (int)((e0 + q) & 3)));
+            return __fadd_rn(lp[q], gumbel(u));
+        };
+        unsigned long long pk0 = 0ull;
+        if (top >= 0) {
+            const float k0 = exact_key(top);
+            if (k0 > -INFINITY) pk0 = pack_key(k0, e0 + top);
+        }
+        best = pk0;
+        const unsigned long long wb = warp_max_u64(pk0);
+        const float B0 = wb ? key_of_pack(wb) : -INFINITY;
+#pragma unroll
+        for (int h = 0; h < kResPer / 4; ++h) {
+            bool any = false;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) any |= (lp[4 * h + i] > -INFINITY && lp[4 * h + i] + kGumbelMax >= B0);
+            if (!any) continue;
+            const uint4 rnd = philox_block(seed, off, kTagResidual, gen_u, (uint64_t)((e0 >> 2) + h));
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int q = 4 * h + i;
+                if (!(lp[q] > -INFINITY) || q == top) continue;
+                const float d = B0 - lp[q];
+                const float u = u01(word_of(rnd, i));
+                if (d > 0.0f) {
+                    const float t = fast_exp2(-d * 1.4426950408889634f);          // exp(-d)
+                    const float ub = fast_exp2(-t * 1.4426950408889634f);         // exp(-exp(-d))
+                    if (u < ub * (1.0f - 1e-4f)) continue;                         // g < d: key below B0
+                }
+                const float key = __fadd_rn(lp[q], gumbel(u));
+                if (key > -INFINITY) {
+                    const unsigned long long pk = pack_key(key, e0 + q);
                     best = pk > best ? pk : best;
                 }
             }

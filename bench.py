@@ -268,6 +268,8 @@ def main(argv=None):
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--workload", default="qwen3_batch")
     ap.add_argument("--e2e-steps", type=int, default=50)
+    ap.add_argument("--copy-streams", type=int, default=2,
+                    help="copy streams sharing the host-to-device copies of the end-to-end measurement")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (a smaller case of the same kernels, for profiling)")
@@ -570,18 +572,33 @@ def main(argv=None):
             sum(x.numel() * x.element_size() for x in (h_T, h_seed, h_off))
         d2h = sum(x.numel() * x.element_size() for x in res)
 
-        # the inputs are copied on two copy streams while the kernels run: the
-        # rows of depth d (and the target rows) on their own, each kernel waiting
-        # only for the copies it reads, each copy waiting only for the previous
-        # step's kernel that reads the same buffer
-        cstreams = [torch.cuda.Stream(device=device), torch.cuda.Stream(device=device)]
-        ev_rows = [torch.cuda.Event() for _ in range(D)]
+        # the inputs are copied while the kernels run, every tensor cut into
+        # row blocks spread over `copy_streams` copy streams (so that several
+        # copy engines share each tensor); each kernel waits only for the copies
+        # it reads, each copy only for the previous step's kernel that read the
+        # same buffer
+        NC = max(1, args.copy_streams)
+        cstreams = [torch.cuda.Stream(device=device) for _ in range(NC)]
+        ev_rows = [[torch.cuda.Event() for _ in range(NC)] for _ in range(D)]
         ev_rows_used = [torch.cuda.Event() for _ in range(D)]
-        ev_small, ev_tgt, ev_step = torch.cuda.Event(), torch.cuda.Event(), torch.cuda.Event()
+        ev_tgt = [torch.cuda.Event() for _ in range(NC)]
+        ev_small, ev_step = torch.cuda.Event(), torch.cuda.Event()
         ev_step.record(stream)
 
+        def split_copy(dst, src, after, done):
+            # rows [i*n/NC, (i+1)*n/NC) of the flattened [rows, V] tensor on stream i
+            d2, s2 = dst.view(-1, dst.shape[-1]), src.view(-1, src.shape[-1])
+            nr = d2.shape[0]
+            for i, cs in enumerate(cstreams):
+                cs.wait_event(after)
+                r0, r1 = nr * i // NC, nr * (i + 1) // NC
+                with torch.cuda.stream(cs):
+                    if r1 > r0:
+                        d2[r0:r1].copy_(s2[r0:r1], non_blocking=True)
+                    done[i].record(cs)
+
         def e2e_step(s):
-            c0, c1 = cstreams
+            c0 = cstreams[0]
             c0.wait_event(ev_step)  # the small inputs are read by every kernel of the step
             with torch.cuda.stream(c0):
                 d_T.copy_(h_T, non_blocking=True)
@@ -589,22 +606,17 @@ def main(argv=None):
                 d_off.copy_(h_off, non_blocking=True)
                 ev_small.record(c0)
             for d in range(D):
-                cs = cstreams[d % 2]
-                cs.wait_event(ev_rows_used[d])
-                with torch.cuda.stream(cs):
-                    d_rows[d].copy_(h_rows[d], non_blocking=True)
-                    ev_rows[d].record(cs)
-            c1.wait_event(ev_step)
-            with torch.cuda.stream(c1):
-                d_tgt.copy_(h_tgt, non_blocking=True)
-                ev_tgt.record(c1)
+                split_copy(d_rows[d], h_rows[d], ev_rows_used[d], ev_rows[d])
+            split_copy(d_tgt, h_tgt, ev_step, ev_tgt)
             s.wait_event(ev_small)
             for d in range(1, D + 1):
-                s.wait_event(ev_rows[d - 1])
+                for e in ev_rows[d - 1]:
+                    s.wait_event(e)
                 rheo.expand(cfg, d, d_rows[d - 1], d_T, d_seed, d_off, tree, ws, s)
                 ev_rows_used[d - 1].record(s)
             rheo.prune(cfg, tree, pr, ws, s)
-            s.wait_event(ev_tgt)
+            for e in ev_tgt:
+                s.wait_event(e)
             rheo.verify(cfg, d_tgt, d_T, d_seed, d_off, tree, pr, out, ws, s)
             for x, h in zip((out.accepted_len, out.accepted_tokens, out.bonus_token), res):
                 h.copy_(x, non_blocking=True)
@@ -624,7 +636,7 @@ def main(argv=None):
             torch.cuda.synchronize()
         e2e_s = reduce_max_time(e0.elapsed_time(e1) / 1e3, world, device)
         e2e = {"value": world * args.e2e_steps / e2e_s, "unit": "tree-steps/s", "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h}
+               "d2h_bytes_per_step": d2h, "copy_streams": NC, "h2d_gbs": h2d * args.e2e_steps / e2e_s / 1e9}
 
     if rank != 0:
         return 0

@@ -187,6 +187,21 @@ def oracle_cycle_seconds(w, draft, reqs):
     return t_build + (time.perf_counter() - t1)
 
 
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu), else the machine type."""
+    import platform
+    import subprocess
+
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return f"{line.split(':', 1)[1].strip()} ({platform.machine()}, {os.cpu_count()} logical CPUs)"
+    except Exception:
+        pass
+    return f"{platform.machine()} ({os.cpu_count()} logical CPUs)"
+
+
 def cpu_baseline(w, draft, budget_s=15.0):
     """The oracle as it stands, on the host cores, over a bounded sample: whole
     cycles of the batch (or of its first requests) repeated for about budget_s."""
@@ -202,7 +217,7 @@ def cpu_baseline(w, draft, budget_s=15.0):
         cycles += 1
     per_step = secs / cycles * w.batch / n
     return {"value": 1.0 / per_step, "unit": "tree-steps/s", "cores": min(cores, max(n, w.K)),
-            "kind": "oracle",
+            "kind": "oracle", "cpu": cpu_model(),
             "sample": f"{cycles} cycles of {n} of {w.batch} requests of {w.name} ({secs:.1f} s), scaled to the full batch"}
 
 
@@ -254,6 +269,7 @@ def run_reference(args, w):
             "config": {"workload": w.name, "batch": w.batch, "vocab": w.vocab, "depth": w.depth, "K": w.K,
                        "budget": w.budget, "logits": w.dtype},
             "cpu_baseline": {"value": value, "unit": "tree-steps/s", "cores": min(cores, w.K), "kind": "oracle",
+                             "cpu": cpu_model(),
                              "sample": f"1 of {w.batch} requests per step, scaled to the full batch"},
             "e2e": {"value": value, "unit": "tree-steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
@@ -670,6 +686,7 @@ def main(argv=None):
                      "frac": ach / peak, "peak_kind": peak_kind, "traffic": traffic,
                      "bytes_per_launch": dom_bytes, "ms_per_launch": dom_ms,
                      "timing": "CUDA events around the depth 2..D launches replayed back to back as in the step"},
+        "request_steps_per_s": world * args.steps / secs * w.batch,
         "kernels": {"expand_ms_per_step": exp_ms, "expand_ms_by_depth": [x / n_k for x in by_depth],
                     "expand_gbs": exp_gbs, "prune_ms": prune_ms,
                     "verify_ms": ver_ms, "verify_gbs": ver_gbs, "step_gbs": step_gbs,

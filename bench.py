@@ -521,7 +521,7 @@ def main(argv=None):
 
         # full support (App. B, Table tab:sparse_support, row Full): the same
         # workload with the sampled token drawn over the whole vocabulary; a graph
-        # of its 12 launches timed like the main step, plus per-call times
+        # of its 14 launches timed like the main step, plus per-call times
         cfg_f = rheo.Config(batch=w.batch, vocab=w.vocab, K=w.K, depth=w.depth, budget=w.budget, m=w.m, support=0,
                             dtype=w.dtype)
         tf, pf, wf = rheo.Tree(cfg_f, device), rheo.Pruned(cfg_f, device), rheo.Workspace(cfg_f, device)
@@ -569,7 +569,7 @@ def main(argv=None):
         full_support = {"tree_steps_per_s": 1e3 / ms_f, "ms_per_step": ms_f,
                         "expand_ms": mk[0].elapsed_time(mk[1]), "prune_ms": mk[1].elapsed_time(mk[2]),
                         "verify_ms": mk[2].elapsed_time(mk[3]),
-                        "note": "eager per-call times; the step time is the CUDA graph of its 12 launches"}
+                        "note": "eager per-call times; the step time is the CUDA graph of its 14 launches"}
 
     # end to end through the public API with host buffers: H2D of every input, D2H of the results
     e2e = None
@@ -697,7 +697,7 @@ def main(argv=None):
                     "full_support": full_support,
                     "tree_attention_bytes": w.batch * (w.budget + 1) * ((w.budget + 1) + 4 + 4 * (w.depth + 1) + 12)},
         "clocks": clocks,
-        "gpu_launches": args.steps * (D + 4),  # D expand, 1 prune, 3 verify (prep, stream, residual)
+        "gpu_launches": args.steps * (D + 5),  # D expand, 1 prune, 4 verify (prep, stream, table, residual)
         "e2e": e2e,
         "cpu_baseline": cpu,
     }

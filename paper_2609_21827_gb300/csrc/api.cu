@@ -47,7 +47,7 @@ bool valid(const rheo_config* c) {
 
 struct Layout {
     size_t status, ex_row_ticket, ex_req_ticket, ex_mu, ex_sum, ex_keys, ex_ltail;
-    size_t v_mu, v_sum, v_row_ticket, v_hdr, v_child, v_tids, v_tq, v_cx, v_tx, v_coin, v_table, v_rhat, r_best,
+    size_t v_mu, v_sum, v_queue, v_hdr, v_child, v_tids, v_tq, v_cx, v_tx, v_coin, v_table, v_rhat, r_best,
         r_ticket;
     size_t total;
 };
@@ -70,7 +70,7 @@ Layout layout(const rheo_config& c) {
     L.ex_ltail = take(2 * sizeof(float) * B * expansions_per_request(c));
     L.v_mu = take(sizeof(float) * B * NP * VC);
     L.v_sum = take(2 * sizeof(float) * B * NP * VC);
-    L.v_row_ticket = take(sizeof(unsigned) * B * NP);
+    L.v_queue = take(sizeof(unsigned));
     L.v_hdr = take(sizeof(int) * B * NP * 8);
     L.v_child = take(sizeof(int) * B * NP * (c.K + 1) * 3);
     L.v_tids = take(sizeof(int) * B * NP * TL);
@@ -277,7 +277,7 @@ extern "C" int rheo_verify_variant(const rheo_config* cfg, int32_t variant, cons
     a.status = at<unsigned>(ws, L.status);
     a.seg_mu = at<float>(ws, L.v_mu);
     a.seg_sum = at<float>(ws, L.v_sum);
-    a.row_ticket = at<unsigned>(ws, L.v_row_ticket);
+    a.queue = at<unsigned>(ws, L.v_queue);
     a.rec_hdr = at<int>(ws, L.v_hdr);
     a.rec_child = at<int>(ws, L.v_child);
     a.rec_tids = at<int>(ws, L.v_tids);
@@ -293,7 +293,6 @@ extern "C" int rheo_verify_variant(const rheo_config* cfg, int32_t variant, cons
     a.n.chunks = verify_chunks_per_row(cfg->dtype == RHEO_BF16 ? 1 : 0, cfg->vocab);
     const int64_t chunks = (int64_t)cfg->batch * NP * a.n.chunks;
     const int grid = verify_stream_grid(sm_count(), chunks);
-    a.units = verify_stream_units(grid, chunks);
     return launch_verify(a, cfg->dtype, rows_aligned(logits, row_stride, *cfg), grid, (cudaStream_t)stream) ==
                    cudaSuccess
                ? RHEO_OK
@@ -338,7 +337,7 @@ extern "C" int rheo_verify_full(const rheo_config* cfg, const void* logits, int6
     a.status = at<unsigned>(ws, L.status);
     a.seg_mu = at<float>(ws, L.v_mu);
     a.seg_sum = at<float>(ws, L.v_sum);
-    a.row_ticket = at<unsigned>(ws, L.v_row_ticket);
+    a.queue = at<unsigned>(ws, L.v_queue);
     a.rec_hdr = at<int>(ws, L.v_hdr);
     a.rec_child = at<int>(ws, L.v_child);
     a.rec_tids = at<int>(ws, L.v_tids);
@@ -354,7 +353,6 @@ extern "C" int rheo_verify_full(const rheo_config* cfg, const void* logits, int6
     a.n.chunks = verify_chunks_per_row(cfg->dtype == RHEO_BF16 ? 1 : 0, cfg->vocab);
     const int64_t chunks = (int64_t)cfg->batch * NP * a.n.chunks;
     const int grid = verify_stream_grid(sm_count(), chunks);
-    a.units = verify_stream_units(grid, chunks);
     return launch_verify_full(a, cfg->dtype, rows_aligned(logits, row_stride, *cfg), draft_aligned, grid,
                               (cudaStream_t)stream) ==
                    cudaSuccess

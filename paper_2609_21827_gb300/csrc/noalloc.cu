@@ -51,7 +51,7 @@ size_t up256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 // the verification part of the workspace layout, laid out in the static array
 struct StaticLayout {
-    size_t status, mu, sum, row_ticket, hdr, child, tids, tq, cx, tx, coin, table, rhat, best, res_ticket, total,
+    size_t status, mu, sum, queue, hdr, child, tids, tq, cx, tx, coin, table, rhat, best, res_ticket, total,
         clear_end;
 };
 
@@ -63,7 +63,7 @@ StaticLayout static_layout(const rheo_config& c) {
     auto take = [&](size_t bytes) { size_t at = o; o = up256(o + bytes); return at; };
     // everything that must start at zero first, so one memset clears it
     L.status = take(sizeof(unsigned));
-    L.row_ticket = take(sizeof(unsigned) * B * NP);
+    L.queue = take(sizeof(unsigned));
     L.best = take(sizeof(unsigned long long) * B * 3);
     L.res_ticket = take(sizeof(unsigned) * B);
     L.clear_end = o;
@@ -146,7 +146,7 @@ extern "C" int rheo_verify_static(const rheo_config* cfg, const void* logits, in
     a.status = reinterpret_cast<unsigned*>(base + L.status);
     a.seg_mu = reinterpret_cast<float*>(base + L.mu);
     a.seg_sum = reinterpret_cast<float*>(base + L.sum);
-    a.row_ticket = reinterpret_cast<unsigned*>(base + L.row_ticket);
+    a.queue = reinterpret_cast<unsigned*>(base + L.queue);
     a.rec_hdr = reinterpret_cast<int*>(base + L.hdr);
     a.rec_child = reinterpret_cast<int*>(base + L.child);
     a.rec_tids = reinterpret_cast<int*>(base + L.tids);
@@ -163,7 +163,6 @@ extern "C" int rheo_verify_static(const rheo_config* cfg, const void* logits, in
         return RHEO_ELAUNCH;
     const int64_t chunks = (int64_t)cfg->batch * (cfg->budget + 1) * a.n.chunks;
     const int grid = verify_stream_grid(sms, chunks);
-    a.units = verify_stream_units(grid, chunks);
     const bool aligned = ((uintptr_t)logits % 16 == 0) && ((row_stride * es) % 16 == 0);
     if (launch_verify(a, cfg->dtype, aligned, grid, s) != cudaSuccess) return RHEO_ELAUNCH;
     if (status && cudaMemcpyAsync(status, base + L.status, sizeof(int32_t), cudaMemcpyDeviceToDevice, s) != cudaSuccess)

@@ -83,7 +83,6 @@ struct VerifyArgs {
     Dims n;                         // n.chunks: 2 KB chunks per target row
     int variant = kVerifyRheo;      // verification rule at every node (kVerify*)
     int prep_grid = 0;              // CTAs of the prep launch (0: one per two rows)
-    int units;                      // warps of the stream launch with work (one contiguous run of chunks each)
     const char* logits;
     int64_t row_stride_bytes;
     const float* T;
@@ -99,7 +98,7 @@ struct VerifyArgs {
     unsigned* status;
     float* seg_mu;                  // [B*(N+1)*chunks]
     float* seg_sum;                 // [B*(N+1)*chunks*2] float-float partition sums
-    unsigned* row_ticket;           // [B*(N+1)] segments of the row streamed so far
+    unsigned* queue;                // [1] grabs of stream units so far (zero between calls)
     int* rec_hdr;                   // [B*(N+1)*8] row records (see verify.cu)
     int* rec_child;                 // [B*(N+1)*(K+1)*3]
     int* rec_tids;                  // [B*(N+1)*TL]
@@ -155,6 +154,5 @@ size_t tree_attn_smem_bytes(int budget);
 int verify_table_width(int K);
 int verify_chunks_per_row(int dtype, int V);
 int verify_stream_grid(int sms, int64_t chunks);
-int verify_stream_units(int grid, int64_t chunks);
 
 }  // namespace rheo

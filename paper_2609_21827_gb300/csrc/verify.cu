@@ -1,19 +1,25 @@
 // verify.cu -- RheoVerification (Algorithm 1) applied layer by layer (Theorem 1).
 //
-// Two launches on the caller's stream:
+// Four launches on the caller's stream:
 //
-// verify_stream_kernel: every warp streams its own contiguous run of 2 KB
-// chunks of the B*(N+1) target rows (16-byte loads straight into registers,
-// the next chunk in flight while the current one is summed), keeping a running
-// (max, sum exp((l - max) / T)) per lane.  Where a row segment of its run ends
-// the warp reduces that state and writes the segment's partial; the warp that
-// ends a row's last segment (arrival counter, never a wait) builds the row's
-// decision table: lse_T from the partials, p at the surviving children and --
-// when the row's sampled child survived -- r^ = max(0, p - q~) over the tail
+// verify_prep_kernel (beside the stream): one warp per pruned row gathers the
+// row's record from the trees (children, tail list, l/T at those tokens, the
+// node's Philox coins).
+//
+// verify_stream_kernel: the B*(N+1) target rows are cut into units of
+// kUnitChunks 2 KB chunks (units never straddle rows); every warp takes units
+// in row order from a counter (its first unit is its index; the next grab is in
+// flight while it streams), loads 16 bytes a lane straight into registers with
+// the next chunk in flight while the current one is summed, and writes one
+// partial (max, sum exp((l - max) / T)) per unit.  Warps that run ahead take
+// more units, so the launch ends when the work does.
+//
+// verify_table_kernel, one warp per pruned row after the stream: the row's
+// decision table -- lse_T from the unit partials, p at the surviving children
+// and, when the row's sampled child survived, r^ = max(0, p - q~) over the tail
 // that child was drawn from, the residual mass M = 1 - sum_tail min(p, q~), r^
-// at the children, the Philox coins of the node, and the verdict of Algorithm
-// 1 at the node.  A row's verdict depends on nothing but the row itself.  The
-// warps never wait for one another.
+// at the children, the node's coins, and the verdict of Algorithm 1 at the
+// node.  A row's verdict depends on nothing but the row itself.
 //
 // residual_kernel, grid (chunks, B): each CTA stages its request's verdicts,
 // replays the walk from the root (a few comparisons per level), and takes part
@@ -40,6 +46,8 @@ __host__ __device__ __forceinline__ int table_width(int K) { return kTabP + 2 * 
 
 constexpr int kCV = 4;                     // 16-byte vectors per lane per chunk
 constexpr int kChunkBytesW = 32 * kCV * 16;  // bytes one warp takes per step
+constexpr int kUnitChunks = 4;             // chunks of one row per stream unit
+__host__ __device__ __forceinline__ int units_per_row(int cpr) { return (cpr + kUnitChunks - 1) / kUnitChunks; }
 
 struct WarpRow {
     int32_t tok[kMaxSupport];   // children slots
@@ -61,15 +69,38 @@ __device__ __forceinline__ int64_t expansion_of_child(int K, int64_t g, int64_t 
     return min((int64_t)parent_expansion_of(K, (int)g), E - 1);
 }
 
-// lse_T of a row from its segment partials (one warp; float-float accumulation)
-__device__ __forceinline__ FF combine_lse(const float* mu, const float* sm, int nseg, float T) {
+// The first 64 unit partials of a row, two per lane, loaded with the row's
+// record so that both arrive in one round trip (absent ones: max -inf, sum 0)
+struct Partials {
+    float mu[2];
+    FF s[2];
+};
+__device__ __forceinline__ Partials load_partials(const float* mu, const float* sm, int nseg) {
     const int lane = threadIdx.x & 31;
-    float m = -INFINITY;
-    for (int c = lane; c < nseg; c += 32) m = fmaxf(m, __ldcg(mu + c));
+    Partials p;
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const int c = lane + 32 * k;
+        const bool ok = c < nseg;
+        p.mu[k] = ok ? __ldcg(mu + c) : -INFINITY;
+        p.s[k] = ok ? FF{__ldcg(sm + 2 * c), __ldcg(sm + 2 * c + 1)} : FF{0.0f, 0.0f};
+    }
+    return p;
+}
+
+// lse_T of a row from its unit partials (one warp; float-float accumulation):
+// the preloaded first 64, the rest (rows of more than 64 units) read here
+__device__ __forceinline__ FF combine_lse(const Partials& p, const float* mu, const float* sm, int nseg, float T) {
+    const int lane = threadIdx.x & 31;
+    float m = fmaxf(p.mu[0], p.mu[1]);
+    for (int c = lane + 64; c < nseg; c += 32) m = fmaxf(m, __ldcg(mu + c));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
     FF t{0.0f, 0.0f};
-    for (int c = lane; c < nseg; c += 32) {
+#pragma unroll
+    for (int k = 0; k < 2; ++k)
+        if (p.s[k].hi != 0.0f) t = ff_add(t, ff_mul(expf(__fdiv_rn(p.mu[k] - m, T)), p.s[k]));
+    for (int c = lane + 64; c < nseg; c += 32) {
         const FF sc{__ldcg(sm + 2 * c), __ldcg(sm + 2 * c + 1)};
         if (sc.hi != 0.0f) t = ff_add(t, ff_mul(expf(__fdiv_rn(__ldcg(mu + c) - m, T)), sc));
     }
@@ -120,10 +151,10 @@ __device__ __forceinline__ void load_chunk(uint4 (&v)[kCV], const char* row, int
 //   cx, tx     l / T as float-float at the children and at the tail tokens
 //   coin       the node's K+2 Philox coins
 constexpr int kHdr = 8;
-// prep runs beside the stream launch: two stream CTAs per SM capped at 96
-// registers a thread leave room for one prep CTA of 256 threads
+// three stream CTAs of 256 threads per SM (more loads in flight per SM than
+// two): 80 registers a thread at most
 constexpr int kPrepThreads = 256;
-constexpr int kStreamMaxRegs = 96;
+constexpr int kStreamMaxRegs = 80;
 
 // One warp per pruned row: the row's record.
 template <int DT>
@@ -225,8 +256,8 @@ __device__ void prep_row(const VerifyArgs& a, int64_t r) {
 }
 
 // One warp per pruned row (the grid may be capped, each warp then taking rows in
-// turn); it runs beside the stream launch and must end before the stream
-// launch's first row finalises, so it keeps one row per warp.
+// turn); it runs beside the stream launch, and the table launch reads its
+// records after the stream launch (which waits for this grid before it ends).
 template <int DT>
 __global__ void __launch_bounds__(kPrepThreads) verify_prep_kernel(const VerifyArgs a) {
     grid_dependency_begin();
@@ -350,9 +381,10 @@ __device__ __noinline__ void finalize_row(const VerifyArgs& a, int64_t r, WarpRo
     const int b = (int)(r / NP);
     const int cpr = n.chunks;
     const int TW = table_width(K);
-    const TileSplit sp{(int64_t)n.B * NP * cpr, a.units};
-    const int nseg = sp.owner(r * cpr + cpr - 1) - sp.owner(r * cpr) + 1;
-    // round trip 1: the record and the partials
+    const int nseg = units_per_row(cpr);
+    // one round trip: the record and the partials
+    const Partials part = load_partials(a.seg_mu + r * cpr, a.seg_sum + 2 * r * cpr, nseg);
+    const float T = a.T[b];
     const int* hdr = a.rec_hdr + r * kHdr;
     const int* child = a.rec_child + r * (K + 1) * 3;
     const int nc = __ldcg(hdr + 0), fc = __ldcg(hdr + 1), sc = __ldcg(hdr + 2);
@@ -373,8 +405,7 @@ __device__ __noinline__ void finalize_row(const VerifyArgs& a, int64_t r, WarpRo
                      : FF{-INFINITY, 0.0f};
     }
     const float coin_l = (lane < K + 2) ? __ldcg(a.rec_coin + r * (K + 2) + lane) : 0.0f;
-    const float T = a.T[b];
-    const FF lse = combine_lse(a.seg_mu + r * cpr, a.seg_sum + 2 * r * cpr, nseg, T);
+    const FF lse = combine_lse(part, a.seg_mu + r * cpr, a.seg_sum + 2 * r * cpr, nseg, T);
     float* tab = a.table + r * TW;
     if (lane == 0) {
         tab[3] = lse.hi;
@@ -465,9 +496,9 @@ __device__ __noinline__ void finalize_row(const VerifyArgs& a, int64_t r, WarpRo
 template <int DT, bool ALIGNED>
 __global__ void __maxnreg__(kStreamMaxRegs) verify_stream_kernel(const VerifyArgs a) {
     // streaming needs nothing from the grids before this one: let the next grid
-    // launch now, and wait for the row records only before the first table
+    // launch now; the wait at the end makes this grid's completion imply the
+    // record launch's
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    __shared__ WarpRow wrs[kWarps];
     using E = Elem<DT>;
     using W = Vec<DT>;
     constexpr int VEC = E::VEC;
@@ -476,74 +507,98 @@ __global__ void __maxnreg__(kStreamMaxRegs) verify_stream_kernel(const VerifyArg
     const Dims& n = a.n;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int V = n.V, NP = n.N + 1;
-    const int cpr = n.chunks;
-    const TileSplit sp{(int64_t)n.B * NP * cpr, a.units};
-    const int u = blockIdx.x * kWarps + warp;
-    if (u >= a.units) return;  // units <= chunks: every unit has at least one chunk
-    const int64_t c0 = sp.begin(u), c1 = sp.begin(u + 1);
-
-    int64_t r = c0 / cpr;
-    int cc = (int)(c0 % cpr);
-    float c = kLog2e / a.T[r / NP];
-    float mu = -INFINITY, sum = 0.0f;
-    uint4 nxt[kCV];
-    load_chunk<DT, ALIGNED>(nxt, a.logits + r * a.row_stride_bytes, cc * CE, V);
-    for (int64_t t = c0; t < c1; ++t, ++cc) {
-        if (cc == cpr) {
-            cc = 0;
-            ++r;
-            c = kLog2e / a.T[r / NP];
-        }
-        const bool seg_last = (t == c1 - 1) || (cc == cpr - 1);
-        uint4 v[kCV];
+    const int cpr = n.chunks, upr = units_per_row(cpr);
+    const int64_t total = (int64_t)n.B * NP * upr;
+    const int64_t nw = (int64_t)gridDim.x * kWarps;
+    // every warp grabs until one grab finds no unit: max(total, nw) grabs in all
+    const int64_t grabs = total > nw ? total : nw;
+    unsigned ticket = 0u;  // lane 0: the grab in flight, read only when needed
+    auto grab = [&]() {
+        if (lane == 0) ticket = atomicAdd(a.queue, 1u);
+    };
+    auto take = [&]() -> int64_t {
+        const unsigned g = __shfl_sync(0xFFFFFFFFu, ticket, 0);
+        if (lane == 0 && (int64_t)g == grabs - 1) atomicExch(a.queue, 0u);  // the last grab: ready for the next call
+        return nw + (int64_t)g;
+    };
+    int64_t q = (int64_t)blockIdx.x * kWarps + warp;  // every warp's first unit is its index
+    grab();
+    if (q >= total) {
+        take();  // the one grab that finds no unit
+    } else {
+        int64_t r = q / upr;
+        int j = (int)(q % upr);
+        float c = kLog2e / a.T[r / NP];
+        uint4 nxt[kCV];
+        load_chunk<DT, ALIGNED>(nxt, a.logits + r * a.row_stride_bytes, j * kUnitChunks * CE, V);
+        for (;;) {
+            const int cc1 = min(cpr, (j + 1) * kUnitChunks);
+            int64_t qn = total, rn = 0;
+            int jn = 0;
+            float cn = 1.0f;
+            float mu = -INFINITY, sum = 0.0f;
+            for (int cc = j * kUnitChunks; cc < cc1; ++cc) {
+                uint4 v[kCV];
 #pragma unroll
-        for (int j = 0; j < kCV; ++j) v[j] = nxt[j];
-        if (t + 1 < c1) {
-            const bool wrap = (cc + 1 == cpr);
-            load_chunk<DT, ALIGNED>(nxt, a.logits + (r + (wrap ? 1 : 0)) * a.row_stride_bytes, wrap ? 0 : (cc + 1) * CE, V);
-        }
-        float tmax = W::vmax(v[0]);
-#pragma unroll
-        for (int j = 1; j < kCV; ++j) tmax = fmaxf(tmax, W::vmax(v[j]));
-        if (tmax > mu) {
-            if (mu != -INFINITY) sum *= fast_exp2((mu - tmax) * c);
-            mu = tmax;
-        }
-        if (mu != -INFINITY) {
-            const float mc = mu * c;
-            float s = 0.0f;
-#pragma unroll
-            for (int j = 0; j < kCV; ++j) s += W::vexp(v[j], c, mc);
-            sum += s;
-        }
-        if (!seg_last) continue;
-        // ---- end of this warp's segment of row r: its partial ------------------
-        float M;
-        const FF Sw = warp_partition(mu, sum, c, M);
-        int last = 0;
-        if (lane == 0) {
-            const int first = sp.owner(r * cpr);
-            const int seg = u - first;
-            const int nseg = sp.owner(r * cpr + cpr - 1) - first + 1;
-            a.seg_mu[r * cpr + seg] = M;
-            a.seg_sum[2 * (r * cpr + seg)] = Sw.hi;
-            a.seg_sum[2 * (r * cpr + seg) + 1] = Sw.lo;
-            if (isnan(Sw.hi) || M == INFINITY) atomicOr(a.status, kStBadLogit);
-            // the warp that ends the row's last segment builds its decision table
-            __threadfence();
-            last = (atomicAdd(a.row_ticket + r, 1u) == (unsigned)nseg - 1u) ? 1 : 0;
-            if (last) {
-                a.row_ticket[r] = 0u;  // ready for the next call
-                __threadfence();
+                for (int k = 0; k < kCV; ++k) v[k] = nxt[k];
+                if (cc + 1 < cc1) {
+                    load_chunk<DT, ALIGNED>(nxt, a.logits + r * a.row_stride_bytes, (cc + 1) * CE, V);
+                } else {  // the unit's last chunk: the next unit's first chunk goes in flight
+                    qn = take();
+                    if (qn < total) {
+                        rn = qn / upr;
+                        jn = (int)(qn % upr);
+                        load_chunk<DT, ALIGNED>(nxt, a.logits + rn * a.row_stride_bytes, jn * kUnitChunks * CE, V);
+                        cn = kLog2e / a.T[rn / NP];
+                    }
+                }
+                float tmax = W::vmax(v[0]);
+        #pragma unroll
+                for (int k = 1; k < kCV; ++k) tmax = fmaxf(tmax, W::vmax(v[k]));
+                if (tmax > mu) {
+                    if (mu != -INFINITY) sum *= fast_exp2((mu - tmax) * c);
+                    mu = tmax;
+                }
+                if (mu != -INFINITY) {
+                    const float mc = mu * c;
+                    float s = 0.0f;
+        #pragma unroll
+                    for (int k = 0; k < kCV; ++k) s += W::vexp(v[k], c, mc);
+                    sum += s;
+                }
             }
+            // the unit's partial, read by the table launch after this grid
+            float M;
+            const FF Sw = warp_partition(mu, sum, c, M);
+            if (lane == 0) {
+                const int64_t at = r * cpr + j;
+                a.seg_mu[at] = M;
+                a.seg_sum[2 * at] = Sw.hi;
+                a.seg_sum[2 * at + 1] = Sw.lo;
+                if (isnan(Sw.hi) || M == INFINITY) atomicOr(a.status, kStBadLogit);
+            }
+            if (qn >= total) break;
+            r = rn;
+            j = jn;
+            c = cn;
+            grab();
         }
-        if (__shfl_sync(0xFFFFFFFFu, last, 0)) {
-            asm volatile("griddepcontrol.wait;" ::: "memory");
-            finalize_row<DT>(a, r, wrs[warp]);
-        }
-        mu = -INFINITY;
-        sum = 0.0f;
     }
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// One warp per pruned row, after the stream launch: the row's decision table.
+template <int DT>
+__global__ void __launch_bounds__(kThreads) verify_table_kernel(const VerifyArgs a) {
+    // the residual launch may queue up now; the partials and records are read
+    // after the wait
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    __shared__ WarpRow wrs[kWarps];
+    const int64_t rows = (int64_t)a.n.B * (a.n.N + 1);
+    const int warp = threadIdx.x >> 5;
+    for (int64_t r = (int64_t)blockIdx.x * kWarps + warp; r < rows; r += (int64_t)gridDim.x * kWarps)
+        finalize_row<DT>(a, r, wrs[warp]);
 }
 
 // ---------------------------------------------------------------------------
@@ -915,6 +970,9 @@ cudaError_t launch_verify_full(const VerifyArgs& a, int dtype, bool aligned, boo
     if (dtype == 1) err = aligned ? go(verify_stream_kernel<1, true>, dim3(grid)) : go(verify_stream_kernel<1, false>, dim3(grid));
     else err = aligned ? go(verify_stream_kernel<0, true>, dim3(grid)) : go(verify_stream_kernel<0, false>, dim3(grid));
     if (err != cudaSuccess) return err;
+    const dim3 gt((unsigned)((rows + kWarps - 1) / kWarps));
+    err = (dtype == 1) ? go(verify_table_kernel<1>, gt) : go(verify_table_kernel<0>, gt);
+    if (err != cudaSuccess) return err;
     const dim3 go_rows((unsigned)rows);
     if (dtype == 1) {
         if (aligned && draft_aligned) err = go(full_overlap_kernel<1, true, true>, go_rows);
@@ -947,6 +1005,10 @@ cudaError_t launch_verify(const VerifyArgs& a, int dtype, bool aligned, int grid
     if (dtype == 1) err = aligned ? go_stream(verify_stream_kernel<1, true>) : go_stream(verify_stream_kernel<1, false>);
     else err = aligned ? go_stream(verify_stream_kernel<0, true>) : go_stream(verify_stream_kernel<0, false>);
     if (err != cudaSuccess) return err;
+    const dim3 gt((unsigned)((rows + kWarps - 1) / kWarps));
+    err = (dtype == 1) ? launch_dependent(verify_table_kernel<1>, gt, dim3(kThreads), 0, s, a)
+                       : launch_dependent(verify_table_kernel<0>, gt, dim3(kThreads), 0, s, a);
+    if (err != cudaSuccess) return err;
     const dim3 g2((a.n.V + kResChunk - 1) / kResChunk, a.n.B);
     if (dtype == 1)
         return aligned ? launch_dependent(residual_kernel<1, true>, g2, dim3(kThreads), 0, s, a)
@@ -960,16 +1022,11 @@ int verify_chunks_per_row(int dtype, int V) {
     const int ce = kChunkBytesW / (dtype == 1 ? 2 : 4);
     return (V + ce - 1) / ce;
 }
-// stream grid: two CTAs per SM, no more CTAs than needed for one chunk per warp
+// stream grid: three CTAs per SM, no more CTAs than needed for one chunk per warp
 int verify_stream_grid(int sms, int64_t chunks) {
-    const int64_t g = 2 * (int64_t)sms;
+    const int64_t g = 3 * (int64_t)sms;
     const int64_t need = (chunks + kWarps - 1) / kWarps;
     return (int)(g < need ? g : need);
-}
-// stream units (warps with work): never more than chunks, so none is empty
-int verify_stream_units(int grid, int64_t chunks) {
-    const int64_t u = (int64_t)grid * kWarps;
-    return (int)(u < chunks ? u : chunks);
 }
 
 }  // namespace rheo

@@ -627,6 +627,7 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     __shared__ uint32_t excl_bits[kResChunk / 32];
     __shared__ uint32_t tail_bits[kResChunk / 32];
     __shared__ int s_stop, s_len;
+    __shared__ unsigned long long s_b0;  // the CTA's best exact key before the filter
     __shared__ int s_path[64];
     __shared__ int s_verdict[kStageRows];
 
@@ -646,6 +647,7 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
         excl_bits[i] = 0u;
         tail_bits[i] = 0u;
     }
+    if (tid == 0) s_b0 = 0ull;
     __syncthreads();
     if (tid == 0) {
         int u = 0, len = 0;
@@ -760,7 +762,7 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
             }
         }
     } else {
-        // key = fp32(lp + g), lp = fp32(l/T - lse).  Exact filter: the warp's best
+        // key = fp32(lp + g), lp = fp32(l/T - lse).  Exact filter: the CTA's best
         // key among each thread's highest-lp token is a lower bound B0 of the
         // winning key; g never exceeds kGumbelMax, so a token with lp + kGumbelMax
         // < B0 cannot win (no uniform drawn); otherwise it can beat B0 only if
@@ -789,7 +791,9 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
         }
         best = pk0;
         const unsigned long long wb = warp_max_u64(pk0);
-        const float B0 = wb ? key_of_pack(wb) : -INFINITY;
+        if ((tid & 31) == 0 && wb) atomicMax(&s_b0, wb);
+        __syncthreads();
+        const float B0 = s_b0 ? key_of_pack(s_b0) : -INFINITY;
 #pragma unroll
         for (int h = 0; h < kResPer / 4; ++h) {
             bool any = false;

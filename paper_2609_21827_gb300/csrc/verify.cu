@@ -536,7 +536,8 @@ __global__ void __maxnreg__(kStreamMaxRegs) verify_stream_kernel(const VerifyArg
             int64_t qn = total, rn = 0;
             int jn = 0;
             float cn = 1.0f;
-            float mu = -INFINITY, sum = 0.0f;
+            float mu = -INFINITY;
+            unsigned long long sum2 = 0ull;  // the running sum as a pair of fp32 partial sums
             for (int cc = j * kUnitChunks; cc < cc1; ++cc) {
                 uint4 v[kCV];
 #pragma unroll
@@ -553,23 +554,27 @@ __global__ void __maxnreg__(kStreamMaxRegs) verify_stream_kernel(const VerifyArg
                     }
                 }
                 float tmax = W::vmax(v[0]);
-        #pragma unroll
+#pragma unroll
                 for (int k = 1; k < kCV; ++k) tmax = fmaxf(tmax, W::vmax(v[k]));
                 if (tmax > mu) {
-                    if (mu != -INFINITY) sum *= fast_exp2((mu - tmax) * c);
+                    if (mu != -INFINITY) {
+                        const float rs = fast_exp2((mu - tmax) * c);
+                        sum2 = f2_mul(sum2, f2_pack(rs, rs));
+                    }
                     mu = tmax;
                 }
-                if (mu != -INFINITY) {
+                if (mu != -INFINITY) {  // packed fp32x2 fma and add, one ex2 per element
                     const float mc = mu * c;
-                    float s = 0.0f;
-        #pragma unroll
-                    for (int k = 0; k < kCV; ++k) s += W::vexp(v[k], c, mc);
-                    sum += s;
+                    const unsigned long long c2 = f2_pack(c, c), n2 = f2_pack(-mc, -mc);
+                    unsigned long long t = W::vexp2(v[0], c2, n2);
+#pragma unroll
+                    for (int k = 1; k < kCV; ++k) t = f2_add(t, W::vexp2(v[k], c2, n2));
+                    sum2 = f2_add(sum2, t);
                 }
             }
             // the unit's partial, read by the table launch after this grid
             float M;
-            const FF Sw = warp_partition(mu, sum, c, M);
+            const FF Sw = warp_partition(mu, f2_fold(sum2), c, M);
             if (lane == 0) {
                 const int64_t at = r * cpr + j;
                 a.seg_mu[at] = M;

@@ -223,8 +223,12 @@ extern "C" int rheo_prune(const rheo_config* cfg, const rheo_tree* tree, const r
     a.tree = tree_ptrs(tree);
     a.pr = pruned_ptrs(pruned);
     a.status = at<unsigned>(ws, L.status);
-    const size_t smem = (sizeof(int32_t) + sizeof(unsigned long long)) * (size_t)a.n.G1 +
-                        5 * sizeof(int32_t) * (size_t)(cfg->budget + 1);
+    size_t smem = (sizeof(int32_t) + sizeof(unsigned long long)) * (size_t)a.n.G1 +
+                  5 * sizeof(int32_t) * (size_t)(cfg->budget + 1);
+    // the nodes' parent, token and slot beside the keys when that still fits
+    const size_t staged = smem + (2 * sizeof(int32_t) + sizeof(uint8_t)) * (size_t)a.n.G1;
+    a.staged = staged <= 160 * 1024 ? 1 : 0;
+    if (a.staged) smem = staged;
     return launch_prune(a, cfg->batch, smem, (cudaStream_t)stream) == cudaSuccess ? RHEO_OK : RHEO_ELAUNCH;
 }
 

@@ -6,6 +6,8 @@
 // ascending (= shallower first, then left to right); the N-th largest key is
 // found by bitwise selection, the survivors are compacted in gen-id order with
 // a block scan, and parents are remapped through a gen -> pruned-index table.
+// When they fit, the nodes' parent, token and slot are read together with the
+// scores, so the kernel makes one round trip to the tree instead of three.
 #include "rheo_device.cuh"
 #include "rheo_kernels.h"
 
@@ -31,9 +33,19 @@ __global__ void __launch_bounds__(kThreads) prune_kernel(const PruneArgs a) {
     int32_t* pfc = ppar + NP;                                                  // [NP] first child
     int32_t* plc = pfc + NP;                                                   // [NP] last child
     int32_t* psc = plc + NP;                                                   // [NP] sampled child
+    int32_t* tpar = psc + NP;                                                  // [G1] parent gen id (staged)
+    int32_t* ttok = tpar + G1;                                                 // [G1] token (staged)
+    uint8_t* tslot = reinterpret_cast<uint8_t*>(ttok + G1);                    // [G1] slot (staged)
+    const bool staged = a.staged != 0;
 
-    for (int g = tid; g < G1; g += kThreads)
+    for (int g = tid; g < G1; g += kThreads) {
         keys[g] = ((unsigned long long)ord_f32(a.tree.score[nb + g]) << 32) | (0xFFFFFFFFu - (uint32_t)g);
+        if (staged) {
+            tpar[g] = a.tree.parent[nb + g];
+            ttok[g] = a.tree.token[nb + g];
+            tslot[g] = a.tree.slot[nb + g];
+        }
+    }
     for (int i = tid; i < NP; i += kThreads) { pfc[i] = -1; plc[i] = -1; psc[i] = -1; }
     __syncthreads();
 
@@ -68,13 +80,13 @@ __global__ void __launch_bounds__(kThreads) prune_kernel(const PruneArgs a) {
         const int g = pgen[i];
         int32_t p = -1;
         if (g != 0) {
-            const int32_t pg = a.tree.parent[nb + g];
+            const int32_t pg = staged ? tpar[g] : a.tree.parent[nb + g];
             p = (pg >= 0 && pg < G1) ? map[pg] : -1;
             if (p < 0) atomicOr(a.status, kStInternal);  // not ancestor-closed (or tree never expanded)
         }
         ppar[i] = p;
         a.pr.gen_id[pb + i] = g;
-        a.pr.token[pb + i] = a.tree.token[nb + g];
+        a.pr.token[pb + i] = staged ? ttok[g] : a.tree.token[nb + g];
         a.pr.depth[pb + i] = depth_of(n.K, g);
         a.pr.parent[pb + i] = p;
     }
@@ -84,7 +96,8 @@ __global__ void __launch_bounds__(kThreads) prune_kernel(const PruneArgs a) {
         if (p < 0) continue;
         if (i == 1 || ppar[i - 1] != p) pfc[p] = i;
         if (i == N || ppar[i + 1] != p) plc[p] = i;
-        if (a.tree.slot[nb + pgen[i]] == kSlotSampled) psc[p] = i;
+        const int g = pgen[i];
+        if ((staged ? tslot[g] : a.tree.slot[nb + g]) == kSlotSampled) psc[p] = i;
     }
     __syncthreads();
     for (int i = tid; i < NP; i += kThreads) {

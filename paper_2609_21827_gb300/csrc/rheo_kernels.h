@@ -64,6 +64,7 @@ struct PruneArgs {
     TreePtrs tree;
     PrunedPtrs pr;
     unsigned* status;
+    int staged;  // parent, token and slot of every node are read with the scores into shared memory
 };
 
 struct TreeAttnArgs {

@@ -68,6 +68,9 @@ SMALL = [
     W("budget1", vocab=700, K=3, depth=3, budget=1, batch=6),
     W("low_T", vocab=5000, K=5, depth=4, budget=15, temperatures=(0.05,), batch=8),
     W("m3_small_support", vocab=3000, K=6, m=3, support=12, depth=3, budget=14, batch=8),
+    # 7906 generated nodes per request: too many for the prune to stage the
+    # nodes' parent, token and slot in shared memory (it reads them from the tree)
+    W("deep_tree", vocab=200, support=64, K=16, depth=30, budget=40, batch=2),
 ]
 
 

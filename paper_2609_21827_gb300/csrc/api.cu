@@ -70,7 +70,7 @@ Layout layout(const rheo_config& c) {
     L.ex_ltail = take(2 * sizeof(float) * B * expansions_per_request(c));
     L.v_mu = take(sizeof(float) * B * NP * VC);
     L.v_sum = take(2 * sizeof(float) * B * NP * VC);
-    L.v_queue = take(sizeof(unsigned));
+    L.v_queue = take(sizeof(unsigned) * kStreamQueues * kStreamQueueStride);
     L.v_hdr = take(sizeof(int) * B * NP * 8);
     L.v_child = take(sizeof(int) * B * NP * (c.K + 1) * 3);
     L.v_tids = take(sizeof(int) * B * NP * TL);

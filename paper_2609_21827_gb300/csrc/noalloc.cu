@@ -63,7 +63,7 @@ StaticLayout static_layout(const rheo_config& c) {
     auto take = [&](size_t bytes) { size_t at = o; o = up256(o + bytes); return at; };
     // everything that must start at zero first, so one memset clears it
     L.status = take(sizeof(unsigned));
-    L.queue = take(sizeof(unsigned));
+    L.queue = take(sizeof(unsigned) * kStreamQueues * kStreamQueueStride);
     L.best = take(sizeof(unsigned long long) * B * 3);
     L.res_ticket = take(sizeof(unsigned) * B);
     L.clear_end = o;

@@ -80,6 +80,10 @@ struct TreeAttnArgs {
 enum : int { kVerifyRheo = 0, kVerifyRrsw = 1, kVerifyOneHot = 2 };
 constexpr int kMaxFullDepth = 32;  // depth limit of full-support verification
 
+// the verification stream's unit counters: kStreamQueues of them, 128 bytes apart
+constexpr int kStreamQueues = 16;
+constexpr int kStreamQueueStride = 32;
+
 struct VerifyArgs {
     Dims n;                         // n.chunks: 2 KB chunks per target row
     int variant = kVerifyRheo;      // verification rule at every node (kVerify*)
@@ -99,7 +103,7 @@ struct VerifyArgs {
     unsigned* status;
     float* seg_mu;                  // [B*(N+1)*chunks]
     float* seg_sum;                 // [B*(N+1)*chunks*2] float-float partition sums
-    unsigned* queue;                // [1] grabs of stream units so far (zero between calls)
+    unsigned* queue;                // [kStreamQueues * kStreamQueueStride] unit counters (zero between calls)
     int* rec_hdr;                   // [B*(N+1)*8] row records (see verify.cu)
     int* rec_child;                 // [B*(N+1)*(K+1)*3]
     int* rec_tids;                  // [B*(N+1)*TL]

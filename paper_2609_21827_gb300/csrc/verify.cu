@@ -8,8 +8,8 @@
 //
 // verify_stream_kernel: the B*(N+1) target rows are cut into units of
 // kUnitChunks 2 KB chunks (units never straddle rows); every warp takes units
-// in row order from a counter (its first unit is its index; the next grab is in
-// flight while it streams), loads 16 bytes a lane straight into registers with
+// in row order from one of kStreamQueues counters (its first unit follows from
+// its index; the next grab is in flight while it streams), loads 16 bytes a lane straight into registers with
 // the next chunk in flight while the current one is summed, and writes one
 // partial (max, sum exp((l - max) / T)) per unit.  Warps that run ahead take
 // more units, so the launch ends when the work does.
@@ -510,18 +510,28 @@ __global__ void __maxnreg__(kStreamMaxRegs) verify_stream_kernel(const VerifyArg
     const int cpr = n.chunks, upr = units_per_row(cpr);
     const int64_t total = (int64_t)n.B * NP * upr;
     const int64_t nw = (int64_t)gridDim.x * kWarps;
-    // every warp grabs until one grab finds no unit: max(total, nw) grabs in all
-    const int64_t grabs = total > nw ? total : nw;
+    // kStreamQueues counters on separate cache lines (one address alone caps the
+    // grab rate): counter k hands out units k, k + Q, k + 2Q, ... (row order) to
+    // the warps w = k mod Q; a warp's first unit is k + Q * (w / Q), its later
+    // ones come from the counter, and every warp grabs until one grab finds no
+    // unit, so counter k sees max(units, warps) grabs of its own in all
+    const int w = blockIdx.x * kWarps + warp;
+    const int qk = w % kStreamQueues;
+    unsigned* ctr = a.queue + qk * kStreamQueueStride;
+    const int64_t nwk = (nw - qk + kStreamQueues - 1) / kStreamQueues;
+    const int64_t tk = total > qk ? (total - qk + kStreamQueues - 1) / kStreamQueues : 0;
+    const int64_t grabs = tk > nwk ? tk : nwk;
     unsigned ticket = 0u;  // lane 0: the grab in flight, read only when needed
     auto grab = [&]() {
-        if (lane == 0) ticket = atomicAdd(a.queue, 1u);
+        if (lane == 0) ticket = atomicAdd(ctr, 1u);
     };
-    auto take = [&]() -> int64_t {
+    auto take = [&]() -> int64_t {  // the next unit, or total when the counter has none left
         const unsigned g = __shfl_sync(0xFFFFFFFFu, ticket, 0);
-        if (lane == 0 && (int64_t)g == grabs - 1) atomicExch(a.queue, 0u);  // the last grab: ready for the next call
-        return nw + (int64_t)g;
+        if (lane == 0 && (int64_t)g == grabs - 1) atomicExch(ctr, 0u);  // its last grab: ready for the next call
+        const int64_t i = nwk + (int64_t)g;
+        return i < tk ? qk + (int64_t)kStreamQueues * i : total;
     };
-    int64_t q = (int64_t)blockIdx.x * kWarps + warp;  // every warp's first unit is its index
+    int64_t q = qk + (int64_t)kStreamQueues * (w / kStreamQueues);
     grab();
     if (q >= total) {
         take();  // the one grab that finds no unit

@@ -275,7 +275,7 @@ __device__ __forceinline__ float exp_ff_minus(FF x, FF c) {
 }
 
 // The decision table of pruned row r (Algorithm 1 at the node), built by one
-// warp from the row's segment partials and its record.
+// warp from the row's unit partials and its record (verify_table_kernel).
 // Vanilla verification of the node's children as a top-K pool (Sec. 2.2,
 // App. A): every surviving child, the sampled one too, a one-hot candidate in
 // slot order against r^ = p; coin draw 1+slot.  Lane 0.

@@ -515,11 +515,13 @@ __global__ void __maxnreg__(kStreamMaxRegs) verify_stream_kernel(const VerifyArg
     // the warps w = k mod Q; a warp's first unit is k + Q * (w / Q), its later
     // ones come from the counter, and every warp grabs until one grab finds no
     // unit, so counter k sees max(units, warps) grabs of its own in all
+    // (Q = min(kStreamQueues, warps), so that every counter has warps)
+    const int Q = nw < kStreamQueues ? (int)nw : kStreamQueues;
     const int w = blockIdx.x * kWarps + warp;
-    const int qk = w % kStreamQueues;
+    const int qk = w % Q;
     unsigned* ctr = a.queue + qk * kStreamQueueStride;
-    const int64_t nwk = (nw - qk + kStreamQueues - 1) / kStreamQueues;
-    const int64_t tk = total > qk ? (total - qk + kStreamQueues - 1) / kStreamQueues : 0;
+    const int64_t nwk = (nw - qk + Q - 1) / Q;
+    const int64_t tk = total > qk ? (total - qk + Q - 1) / Q : 0;
     const int64_t grabs = tk > nwk ? tk : nwk;
     unsigned ticket = 0u;  // lane 0: the grab in flight, read only when needed
     auto grab = [&]() {
@@ -529,9 +531,9 @@ __global__ void __maxnreg__(kStreamMaxRegs) verify_stream_kernel(const VerifyArg
         const unsigned g = __shfl_sync(0xFFFFFFFFu, ticket, 0);
         if (lane == 0 && (int64_t)g == grabs - 1) atomicExch(ctr, 0u);  // its last grab: ready for the next call
         const int64_t i = nwk + (int64_t)g;
-        return i < tk ? qk + (int64_t)kStreamQueues * i : total;
+        return i < tk ? qk + (int64_t)Q * i : total;
     };
-    int64_t q = qk + (int64_t)kStreamQueues * (w / kStreamQueues);
+    int64_t q = qk + (int64_t)Q * (w / Q);
     grab();
     if (q >= total) {
         take();  // the one grab that finds no unit

@@ -71,6 +71,9 @@ SMALL = [
     # 7906 generated nodes per request: too many for the prune to stage the
     # nodes' parent, token and slot in shared memory (it reads them from the tree)
     W("deep_tree", vocab=200, support=64, K=16, depth=30, budget=40, batch=2),
+    # the largest vocabulary the library accepts (262,144), in both dtypes
+    W("max_vocab_bf16", vocab=262144, dtype="bf16", K=4, depth=2, budget=8, batch=2),
+    W("max_vocab_f32", vocab=262144, K=4, depth=2, budget=8, batch=2, temperatures=(0.6,)),
 ]
 
 

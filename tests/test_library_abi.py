@@ -47,7 +47,8 @@ def test_sizes_of_the_workloads(lib, name):
 @pytest.mark.parametrize("bad", [dict(m=5, K=4), dict(support=4, K=4), dict(budget=0), dict(budget=10**6),
                                  dict(K=0, depth=2), dict(m=0, eps=0.0), dict(vocab=300000), dict(vocab=262145),
                                  dict(dtype="f16"),
-                                 dict(K=127, depth=3), dict(batch=70000)])
+                                 dict(K=127, depth=3), dict(batch=70000), dict(batch=0), dict(vocab=0),
+                                 dict(depth=0), dict(K=-1), dict(m=-1), dict(support=129, K=4)])
 def test_invalid_configurations_are_rejected(lib, bad):
     # (the largest vocabulary accepted is 262,144; tests/test_gpu_parity.py runs it)
     base = dict(batch=2, vocab=1000, K=4, depth=3, budget=10, m=1)

@@ -11,7 +11,10 @@
 // The array is a static device variable: every GPU that loads this library
 // holds its kStaticScratchBytes until the process exits.  Its device address is
 // looked up once per device, by the first call made on that device (with that
-// device current); make that first call before any stream capture.  All calls
+// device current); make that first call before any stream capture.  The address
+// is cached for the life of the process: it does not survive a
+// cudaDeviceReset (or any other teardown of the device's primary context), after
+// which this entry point must not be called again in the same process.  All calls
 // share the array and it keeps the last call's contents, so calls whose work
 // overlaps on the GPU (other streams, other threads) race on it: serialise them.
 #include <cuda_runtime.h>
@@ -115,6 +118,8 @@ extern "C" int rheo_verify_static(const rheo_config* cfg, const void* logits, in
     if (cudaMemsetAsync(base, 0, L.clear_end, s) != cudaSuccess) return RHEO_ELAUNCH;
 
     VerifyArgs a;
+    a.n = Dims{};
+    a.n.full = 0;  // sparse support only (full support is refused above)
     a.n.B = cfg->batch;
     a.n.V = cfg->vocab;
     a.n.K = cfg->K;

@@ -31,13 +31,13 @@ struct PrunedPtrs {
 };
 
 struct Dims {
-    int B, V, K, m, S, D, N;
-    int full;    // full support: S = K+1 ranks selected, the sampled token drawn over V
-    int TL;      // S - m
-    int GW;      // gathered logits per verify row: (K+1) + TL
-    int chunks;  // chunks per row
-    int64_t G1, E;
-    float eps;
+    int B = 0, V = 0, K = 0, m = 0, S = 0, D = 0, N = 0;
+    int full = 0;    // full support: S = K+1 ranks selected, the sampled token drawn over V
+    int TL = 0;      // S - m
+    int GW = 0;      // gathered logits per verify row: (K+1) + TL
+    int chunks = 0;  // chunks per row
+    int64_t G1 = 0, E = 0;
+    float eps = 0.0f;
 };
 
 struct ExpandArgs {

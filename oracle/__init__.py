@@ -43,6 +43,8 @@ def build(force: bool = False) -> str:
 
 
 VERIFY_RHEO, VERIFY_RRSW, VERIFY_ONEHOT = 0, 1, 2
+# mistakes planted on purpose (tests that must reject them); see rheo_oracle.h
+PLANT_NONE, PLANT_RESIDUAL_ON_SUPPORT, PLANT_MASS_ON_SUPPORT = 0, 1, 2
 
 
 class _Cfg(ctypes.Structure):
@@ -51,7 +53,7 @@ class _Cfg(ctypes.Structure):
         ("m", ctypes.c_int32), ("S", ctypes.c_int32), ("D", ctypes.c_int32),
         ("N", ctypes.c_int32), ("eps", ctypes.c_double),
         ("proxy_mode", ctypes.c_int32), ("fixed_log_proxy", ctypes.c_double),
-        ("verify_mode", ctypes.c_int32),
+        ("verify_mode", ctypes.c_int32), ("plant_mode", ctypes.c_int32),
     ]
 
 
@@ -127,6 +129,7 @@ class Config:
     proxy_mode: int = 0
     fixed_log_proxy: float = 0.0
     verify_mode: int = 0  # VERIFY_RHEO, VERIFY_RRSW or VERIFY_ONEHOT
+    plant_mode: int = 0   # PLANT_*: tests only
 
     def __post_init__(self):
         if self.S is None:
@@ -134,7 +137,7 @@ class Config:
 
     def c(self) -> _Cfg:
         return _Cfg(self.B, self.V, self.K, self.m, self.S, self.D, self.N, self.eps,
-                    self.proxy_mode, self.fixed_log_proxy, self.verify_mode)
+                    self.proxy_mode, self.fixed_log_proxy, self.verify_mode, self.plant_mode)
 
     @property
     def G1(self) -> int:

@@ -60,6 +60,7 @@ int orc_check_cfg(const orc_cfg* c) {
     if (c->N < 1 || c->N > G1 - 1) return -1;
     if (c->m == 0 && !(c->eps > 0.0)) return -1;
     if (c->verify_mode < ORC_VERIFY_RHEO || c->verify_mode > ORC_VERIFY_ONEHOT) return -1;
+    if (c->plant_mode < ORC_PLANT_NONE || c->plant_mode > ORC_PLANT_MASS_ON_SUPPORT) return -1;
     return 0;
 }
 
@@ -607,6 +608,7 @@ static int verify_request(const orc_cfg* c, int b, const float* target, float T,
         double M = 1.0;
         int use_tail = 0;
         const int32_t* tids = NULL;
+        int64_t pool0 = -1; /* gen id of slot 0 in the pool of u's sampled child (after its rejection) */
         int accepted = -1;
         if (c->verify_mode != ORC_VERIFY_RHEO) {
             accepted = verify_variant(c, b, l, lu, T, seed, offset, t, p, u, gl + len, rhat, tail_pos, &tids,
@@ -637,6 +639,12 @@ static int verify_request(const orc_cfg* c, int b, const float* target, float T,
                     }
                     M = 1.0 - overlap;
                     use_tail = 1;
+                    pool0 = gs - c->m;
+                    if (c->plant_mode == ORC_PLANT_MASS_ON_SUPPORT) {
+                        M = 0.0;
+                        for (int i = 0; i < TL; ++i) M += (double)rhat[i];
+                        for (int j = 0; j < c->m; ++j) M += (double)P_OF(t->token[nb + pool0 + j]);
+                    }
                 }
             }
             if (accepted < 0 && nc > 0) {
@@ -678,6 +686,11 @@ static int verify_request(const orc_cfg* c, int b, const float* target, float T,
                 for (int k = 0; k < nc && pass < 2; ++k)
                     if (p->token[pb + fc + k] == v) { excluded = 1; break; }
                 if (excluded) continue;
+                if (pass == 0 && use_tail && c->plant_mode == ORC_PLANT_RESIDUAL_ON_SUPPORT && tail_pos[v] < 0) {
+                    int lead = 0;
+                    for (int j = 0; j < c->m; ++j) lead |= (t->token[nb + pool0 + j] == v);
+                    if (!lead) continue;
+                }
                 const float g = gumbel(orc_uniform(seed, offset, ORC_TAG_RESIDUAL, (int32_t)gu, (uint64_t)v));
                 const float tv = l[v] / T;
                 float key;

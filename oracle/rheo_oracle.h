@@ -47,7 +47,20 @@ typedef struct {
     int32_t proxy_mode;      /* 0: the paper's proxy. 1: fixed log-proxy (planted mistake for tests) */
     double fixed_log_proxy;  /* used only when proxy_mode == 1 */
     int32_t verify_mode;     /* ORC_VERIFY_*: the verification rule applied at every node */
+    int32_t plant_mode;      /* ORC_PLANT_*: a mistake planted on purpose, for tests that must
+                                reject it; 0 everywhere else */
 } orc_cfg;
+
+/* Planted mistakes in Algorithm 1 after the sampled child is rejected (test
+ * infrastructure: each is a no-op when the support covers the vocabulary, so
+ * only tests at S < V can tell them from the method):
+ *  RESIDUAL_ON_SUPPORT  the final draw u* ~ r^ considers only the expansion's
+ *                       support (its m leads and its tail), dropping r^ = p
+ *                       off the support;
+ *  MASS_ON_SUPPORT      the residual mass M is summed over the support only
+ *                       (tail r^ plus p at the leads) instead of
+ *                       1 - sum_tail min(p, q~). */
+enum { ORC_PLANT_NONE = 0, ORC_PLANT_RESIDUAL_ON_SUPPORT = 1, ORC_PLANT_MASS_ON_SUPPORT = 2 };
 
 /* Verification rules (all lossless):
  *  RHEO    Algorithm 1: the sampled child first (accept iff eta*q~ <= p), then

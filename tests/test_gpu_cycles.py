@@ -66,6 +66,34 @@ def test_first_two_tokens_follow_the_target(variant, m, T):
     assert _chisq_p(counts, law * counts.sum()) > 0.01
 
 
+@pytest.mark.parametrize("variant", [rheo.VERIFY_RHEO, rheo.VERIFY_RRSW, rheo.VERIFY_ONEHOT])
+@pytest.mark.parametrize("m,S,T", [(1, 12, 1.0), (0, 8, 0.7), (2, 10, 1.3)])
+def test_first_two_tokens_follow_the_target_sparse_support(variant, m, S, T):
+    """Support S < V (Sec. 3.2 "Efficient implementation"): the sampled token
+    comes from the truncated tail and verification uses the same truncated q~;
+    the residual off the support is p.  The emitted stream must still follow
+    the target exactly."""
+    V, k, B = 24, 1, 6000
+    draft, target = _models(V, k, seed=300 + m + S)
+    cfg = rheo.Config(batch=B, vocab=V, K=3, depth=3, budget=8, m=m, support=S, dtype="f32")
+    counts = np.zeros(V * V)
+    for rep in range(2):
+        window = torch.full((B, k), 5, dtype=torch.int64, device="cuda")
+        seed = torch.arange(B, dtype=torch.int64, device="cuda") * 6007 + 1000033 * rep + 29
+        res = cycles.run_cycles(cfg, draft, target, window, torch.full((B,), T), seed, cycles=2, L=2,
+                                variant=variant)
+        st = res.streams.cpu().numpy()
+        assert (st >= 0).all()
+        counts += np.bincount(st[:, 0] * V + st[:, 1], minlength=V * V)
+    tab = target.table.cpu().double().numpy() / T
+    p1 = np.exp(tab[5] - tab[5].max()); p1 /= p1.sum()
+    law = np.zeros(V * V)
+    for a in range(V):
+        p2 = np.exp(tab[a] - tab[a].max()); p2 /= p2.sum()
+        law[a * V:(a + 1) * V] = p1[a] * p2
+    assert _chisq_p(counts, law * counts.sum()) > 0.01
+
+
 def _thm2(p, order, qt, n):
     """App. D.1: acceptance of one layer of n = K+1 slots with nothing pruned."""
     top = order[: n - 1]
@@ -76,11 +104,12 @@ def _thm2(p, order, qt, n):
             + r[order[n - 1]] * sum(max(0.0, qt[v] - p[v]) for v in top))
 
 
-@pytest.mark.parametrize("K,m,T", [(2, 1, 1.0), (3, 1, 0.7), (3, 0, 1.0)])
-def test_single_layer_acceptance_matches_theorem2_across_cycles(K, m, T):
+@pytest.mark.parametrize("K,m,T,S", [(2, 1, 1.0, 24), (3, 1, 0.7, 24), (3, 0, 1.0, 24), (2, 1, 1.0, 12),
+                                     (3, 0, 0.8, 8)])
+def test_single_layer_acceptance_matches_theorem2_across_cycles(K, m, T, S):
     V, k, B, C = 24, 1, 4000, 6
     draft, target = _models(V, k, seed=200 + K + m, noise=1.0)
-    cfg = rheo.Config(batch=B, vocab=V, K=K, depth=1, budget=K + 1, m=m, support=V, dtype="f32")
+    cfg = rheo.Config(batch=B, vocab=V, K=K, depth=1, budget=K + 1, m=m, support=S, dtype="f32")
     window = torch.randint(0, V, (B, k), generator=torch.Generator().manual_seed(5)).cuda()
     seed = torch.arange(B, dtype=torch.int64, device="cuda") * 104729 + 11
     res = cycles.run_cycles(cfg, draft, target, window, torch.full((B,), T), seed, cycles=C, L=1)
@@ -92,10 +121,10 @@ def test_single_layer_acceptance_matches_theorem2_across_cycles(K, m, T):
     for ctx in range(V):
         row = dtab[ctx]
         order = sorted(range(V), key=lambda v: (-row[v], v))
-        qt = np.zeros(V)
-        t = row[order[m:]] / T
+        qt = np.zeros(V)  # q~ over the tail: support ranks m+1..S
+        t = row[order[m:S]] / T
         e = np.exp(t - t.max())
-        qt[order[m:]] = e / e.sum()
+        qt[order[m:S]] = e / e.sum()
         pt = np.exp(ttab[ctx] / T - (ttab[ctx] / T).max())
         pt /= pt.sum()
         expect[ctx] = _thm2(pt, order, qt, K + 1)

@@ -334,15 +334,18 @@ def _thm2(p, order, qt, n):
             + r[order[n - 1]] * sum(max(0.0, qt[v] - p[v]) for v in top_nm1))
 
 
-@pytest.mark.parametrize("V,K,m,T", [(8, 2, 1, 1.0), (9, 3, 1, 0.7), (8, 3, 2, 1.0), (7, 2, 0, 1.3)])
-def test_theorem2_single_layer_acceptance(orc, V, K, m, T):
-    dr, tg, en, p, order, qt = _single_layer(V, K, m, K + 1, T, seed=V * 7 + K)
+@pytest.mark.parametrize("V,K,m,T,S", [(8, 2, 1, 1.0, 8), (9, 3, 1, 0.7, 9), (8, 3, 2, 1.0, 8), (7, 2, 0, 1.3, 7),
+                                       (8, 2, 1, 1.0, 5), (10, 2, 1, 0.8, 4), (7, 2, 0, 1.3, 4)])
+def test_theorem2_single_layer_acceptance(orc, V, K, m, T, S):
+    """App. D.1 closed form (q~ truncated to the support when S < V) against
+    the enumerator and 2*10^5 oracle cycles."""
+    dr, tg, en, p, order, qt = _single_layer(V, K, m, K + 1, T, seed=V * 7 + K, S=S)
     want = _thm2(p, order, qt, K + 1)
     _, acc = en.stream_distribution(1)
     assert abs(acc[1] - want) < 1e-12
     upper = sum(p[v] for v in order[: K + 1]) + sum(min(p[v], qt[v]) for v in order[K + 1:])
     assert want <= upper + 1e-15
-    cfg = orc.Config(B=1, V=V, K=K, m=m, D=1, N=K + 1)
+    cfg = orc.Config(B=1, V=V, K=K, m=m, S=S, D=1, N=K + 1)
     n = 200000
     _, a = orc.run_prefix_lm(cfg, dr, tg, 1, n, T, 999, 1)
     assert abs(a.mean() - want) <= 5 * math.sqrt(want * (1 - want) / n) + 1e-12
@@ -428,6 +431,69 @@ def test_monte_carlo_detects_planted_proxy_mistake(orc):
     bad = orc.Config(B=1, V=3, K=2, m=1, D=1, N=2, proxy_mode=1, fixed_log_proxy=math.log(0.25))
     st, _ = orc.run_prefix_lm(bad, dr, tg, 1, n, 1.0, 1, 1)
     assert _chisq_p(np.bincount(st[:, 0], minlength=3), pt * n) < 1e-6
+
+
+# --------------------------------------------------------------------------
+# sparse support S < V (Sec. 3.2 "Efficient implementation": verification with
+# the same truncated q~ stays lossless).  Only here does the residual off the
+# support (r^ = p there) and the mass M = 1 - sum_tail min(p, q~) take part.
+# --------------------------------------------------------------------------
+
+def _sparse_laws(V, K, m, S, D, N, T, seed):
+    rng = np.random.default_rng(seed)
+    dr, tg = bf.random_tables(rng, V, D)
+    en = bf.Enumerator(V, K, m, S, D, N, T, dr, tg)
+    tl = en.target_law(2)
+    p1 = np.zeros(V)
+    p2 = np.zeros(V * V)
+    for (a, b), pr in tl.items():
+        p1[a] += pr
+        p2[a * V + b] += pr
+    _, accl = en.stream_distribution(2)
+    return dr, tg, p1, p2, np.array([accl.get(i, 0.0) for i in range(D + 1)])
+
+
+SPARSE_MC = [(8, 0), (8, 1), (8, 2), (12, 0), (12, 1), (12, 2)]
+
+
+@pytest.mark.parametrize("S,m", SPARSE_MC)
+def test_monte_carlo_losslessness_sparse_support(orc, S, m):
+    """10^6 oracle cycles at V = 16 with support S < V: the first emitted token
+    and the first two follow the target (Theorem 1), and the accepted length
+    follows the enumerator's exact law, which forms the residual as
+    max(0, p - q~) over the whole vocabulary (q~ = 0 off the tail)."""
+    V, K, D, N, T, n = 16, 2, 2, 5, 0.9, 1_000_000
+    dr, tg, p1, p2, ea = _sparse_laws(V, K, m, S, D, N, T, seed=1700 + 10 * S + m)
+    cfg = orc.Config(B=1, V=V, K=K, m=m, S=S, D=D, N=N)
+    st, acc = orc.run_prefix_lm(cfg, dr, tg, D, n, T, 4242 + S + m, 2)
+    assert _chisq_p(np.bincount(st[:, 0], minlength=V), p1 * n) > 0.01
+    assert _chisq_p(np.bincount(st[:, 0] * V + st[:, 1], minlength=V * V), p2 * n) > 0.01
+    assert _chisq_p(np.bincount(acc, minlength=D + 1), ea * n) > 0.01
+
+
+@pytest.mark.parametrize("plant", ["residual_on_support", "mass_on_support"])
+def test_monte_carlo_detects_planted_sparse_support_mistakes(orc, plant):
+    """Two plausible mistakes planted in the oracle (restricting the final draw
+    to the expansion's support; summing the residual mass over the support
+    only) are invisible at S = V, where the support is the whole vocabulary,
+    and the chi-square tests above reject each of them at S < V."""
+    mode = {"residual_on_support": orc.PLANT_RESIDUAL_ON_SUPPORT, "mass_on_support": orc.PLANT_MASS_ON_SUPPORT}[plant]
+    V, K, m, D, N, T, n = 16, 2, 1, 2, 5, 0.9, 400_000
+    for S, must_pass in ((V, True), (8, False)):
+        dr, tg, p1, p2, ea = _sparse_laws(V, K, m, S, D, N, T, seed=1900 + S)
+        clean = orc.Config(B=1, V=V, K=K, m=m, S=S, D=D, N=N)
+        bad = orc.Config(B=1, V=V, K=K, m=m, S=S, D=D, N=N, plant_mode=mode)
+        st0, acc0 = orc.run_prefix_lm(clean, dr, tg, D, n, T, 99, 2)
+        st1, acc1 = orc.run_prefix_lm(bad, dr, tg, D, n, T, 99, 2)
+        pv = min(_chisq_p(np.bincount(st1[:, 0] * V + st1[:, 1], minlength=V * V), p2 * n),
+                 _chisq_p(np.bincount(acc1, minlength=D + 1), ea * n))
+        if must_pass:
+            # same draws, and the planted branch is never taken differently
+            np.testing.assert_array_equal(st0, st1)
+            np.testing.assert_array_equal(acc0, acc1)
+        else:
+            assert _chisq_p(np.bincount(st0[:, 0] * V + st0[:, 1], minlength=V * V), p2 * n) > 0.01
+            assert pv < 1e-6, (plant, pv)
 
 
 # --------------------------------------------------------------------------

@@ -74,16 +74,17 @@ class Clocks:
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, interval_ms: int = 20):
         self.path = tempfile.mktemp(prefix="rheo_clocks_", suffix=".csv")
         self.proc = None
         self.gpu = gpu_index
+        self.interval_ms = interval_ms
 
     def __enter__(self):
         try:
             self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                          "--format=csv,noheader,nounits", "-lms", str(self.interval_ms)],
                                          stdout=self.fh, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
@@ -152,11 +153,12 @@ def barrier(world: int):
         dist.barrier()
 
 
-def oracle_cycle_seconds(w, draft, reqs):
-    """Seconds of one CPU-oracle cycle on requests `reqs` of the workload inputs.
+def oracle_cycle(w, draft, reqs):
+    """One CPU-oracle cycle on requests `reqs` of the workload inputs.
 
     Expansion and prune are timed, target rows are built (untimed) from the
-    oracle's own pruned tree, then verification is timed."""
+    oracle's own pruned tree, then verification is timed.  Returns the seconds
+    and the oracle's tree, pruned tree and verification outputs."""
     import numpy as np
     import torch
 
@@ -183,8 +185,75 @@ def oracle_cycle_seconds(w, draft, reqs):
     tgt = synth.target_rows(w, sub, [torch.from_numpy(f) for f in frontiers], torch.from_numpy(pr.gen_id.copy()),
                             request_ids=reqs).float().cpu().numpy()
     t1 = time.perf_counter()
-    oracle.verify(ocfg, tgt, T, seed, off, tree, pr)
-    return t_build + (time.perf_counter() - t1)
+    out = oracle.verify(ocfg, tgt, T, seed, off, tree, pr)
+    return t_build + (time.perf_counter() - t1), tree, pr, out
+
+
+PRUNED_FIELDS = ("gen_id", "token", "parent", "depth", "first_child", "n_child", "sampled_child")
+FLIP_GAP = 1e-6
+
+
+def gpu_outputs(tree, pr, out):
+    """Host copies of the integer results of a GPU cycle (for the parity report)."""
+    g = {k: getattr(tree, k).cpu().numpy() for k in ("token", "parent", "slot")}
+    g.update({"pr_" + k: getattr(pr, k).cpu().numpy() for k in PRUNED_FIELDS})
+    g.update(acc_len=out.accepted_len.cpu().numpy(), acc_tok=out.accepted_tokens.cpu().numpy(),
+             acc_node=out.accepted_nodes.cpu().numpy(), bonus=out.bonus_token.cpu().numpy())
+    return g
+
+
+def parity_summary(w, g, reqs, ot, op, oo):
+    """GPU against oracle on requests `reqs`: every integer result compared
+    bit for bit (trees depth by depth, the pruned tree, the accepted path and
+    the bonus token).  A request that differs is an explained near-tie flip
+    when the oracle's relative margin at the first divergent decision is below
+    FLIP_GAP, else unexplained."""
+    import numpy as np
+
+    K, D = w.K, w.depth
+    exact, flips, bad = 0, [], []
+    for j, b in enumerate(reqs):
+        why = None
+        for d in range(1, D + 1):
+            F = 1 if d == 1 else K
+            base = 1 if d == 1 else 1 + (K + 1) + (d - 2) * K * (K + 1)
+            sl = slice(base, base + F * (K + 1))
+            if d >= 2 and not np.array_equal(g["parent"][b, sl], ot.parent[j, sl]):
+                why = ("frontier", float(ot.gap_frontier[j, d - 2]))
+            elif not np.array_equal(g["token"][b, sl], ot.token[j, sl]):
+                for f in range(F):
+                    ps = slice(base + f * (K + 1), base + (f + 1) * (K + 1))
+                    if not np.array_equal(g["token"][b, ps], ot.token[j, ps]):
+                        e = 0 if d == 1 else 1 + (d - 2) * K + f
+                        why = ("sample", float(ot.gap_sample[j, e]))
+                        break
+            elif not np.array_equal(g["slot"][b, sl], ot.slot[j, sl]):
+                why = ("pool", 1.0)
+            if why:
+                break
+        if why is None and not np.array_equal(g["pr_gen_id"][b], op.gen_id[j]):
+            why = ("prune", float(op.gap_prune[j]))
+        if why is None and any(not np.array_equal(g["pr_" + k][b], getattr(op, k)[j]) for k in PRUNED_FIELDS):
+            why = ("pruned_fields", 1.0)
+        if why is None:
+            lvl = None
+            for i in range(D):
+                if g["acc_node"][b, i] != oo.accepted_nodes[j, i] or g["acc_tok"][b, i] != oo.accepted_tokens[j, i]:
+                    lvl = i
+                    break
+            if lvl is None and (g["acc_len"][b] != oo.accepted_len[j] or g["bonus"][b] != oo.bonus_token[j]):
+                lvl = min(int(oo.accepted_len[j]), int(g["acc_len"][b]))
+            if lvl is not None:
+                why = ("verify", float(oo.gap_level[j, lvl]))
+        if why is None:
+            exact += 1
+        elif why[1] < FLIP_GAP:
+            flips.append({"request": int(b), "at": why[0], "gap": why[1]})
+        else:
+            bad.append({"request": int(b), "at": why[0], "gap": why[1]})
+    return {"requests": len(reqs), "exact": exact, "explained_flips": len(flips), "unexplained": len(bad),
+            "flips": flips, "mismatches": bad[:8], "flip_gap": FLIP_GAP,
+            "compared": "tree tokens, parents and slots at every depth, pruned tree, accepted path, bonus token"}
 
 
 def cpu_model() -> str:
@@ -202,23 +271,44 @@ def cpu_model() -> str:
     return f"{platform.machine()} ({os.cpu_count()} logical CPUs)"
 
 
-def cpu_baseline(w, draft, budget_s=15.0):
+def cpu_baseline(w, draft, gpu=None, budget_s=12.0, budget_1t_s=6.0):
     """The oracle as it stands, on the host cores, over a bounded sample: whole
-    cycles of the batch (or of its first requests) repeated for about budget_s."""
+    cycles of the batch (or of its first requests) repeated for about budget_s
+    with every core, then cycles of single requests on one thread for about
+    budget_1t_s.  With `gpu` (the GPU's results of the same inputs), the last
+    all-core cycle's results are also compared with them (parity report)."""
     import oracle
 
     oracle.build()
-    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
-    first = oracle_cycle_seconds(w, draft, [0])
+    threads0 = oracle.max_threads()
+    first, *_ = oracle_cycle(w, draft, [0])
     n = max(1, min(w.batch, int(budget_s / max(first, 1e-3))))
-    secs, cycles = 0.0, 0
+    oracle.threads_used(reset=True)
+    secs, cycles, last = 0.0, 0, None
     while cycles == 0 or (secs < budget_s * 0.7 and cycles < 50):
-        secs += oracle_cycle_seconds(w, draft, range(n)) if n > 1 else first
+        t, *last = oracle_cycle(w, draft, range(n))
+        secs += t
         cycles += 1
+    used = oracle.threads_used(reset=True)
     per_step = secs / cycles * w.batch / n
-    return {"value": 1.0 / per_step, "unit": "tree-steps/s", "cores": min(cores, max(n, w.K)),
-            "kind": "oracle", "cpu": cpu_model(),
-            "sample": f"{cycles} cycles of {n} of {w.batch} requests of {w.name} ({secs:.1f} s), scaled to the full batch"}
+    # one thread: single requests in turn
+    oracle.set_threads(1)
+    secs1, cyc1 = 0.0, 0
+    try:
+        while cyc1 == 0 or (secs1 < budget_1t_s and cyc1 < 4 * w.batch):
+            t, *_ = oracle_cycle(w, draft, [cyc1 % w.batch])
+            secs1 += t
+            cyc1 += 1
+        used1 = oracle.threads_used(reset=True)
+    finally:
+        oracle.set_threads(threads0)
+    base = {"value": 1.0 / per_step, "unit": "tree-steps/s", "cores": used, "kind": "oracle", "cpu": cpu_model(),
+            "sample": f"{cycles} cycles of {n} of {w.batch} requests of {w.name} ({secs:.1f} s), scaled to the "
+                      f"full batch; cores = OpenMP threads that ran part of the oracle's loops",
+            "one_thread": {"value": 1.0 / (secs1 / cyc1 * w.batch), "unit": "tree-steps/s", "cores": used1,
+                           "sample": f"{cyc1} cycles of single requests ({secs1:.1f} s), scaled to the full batch"}}
+    par = parity_summary(w, gpu, list(range(n)), *last) if gpu is not None else None
+    return base, par
 
 
 def build_inputs(w, device):
@@ -256,21 +346,23 @@ def run_reference(args, w):
     device = "cuda" if torch.cuda.is_available() else "cpu"
     draft = synth.make_draft_inputs(w, device=device)
     times = []
+    oracle.threads_used(reset=True)
     for i in range(args.warmup + args.steps):
-        t = oracle_cycle_seconds(w, draft, [i % w.batch])
+        t, *_ = oracle_cycle(w, draft, [i % w.batch])
         if i >= args.warmup:
             times.append(t * w.batch)
     per_step = sum(times) / len(times)
-    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    cores = oracle.threads_used(reset=True)
     value = 1.0 / per_step
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tree-steps/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_step * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": w.name, "batch": w.batch, "vocab": w.vocab, "depth": w.depth, "K": w.K,
                        "budget": w.budget, "logits": w.dtype},
-            "cpu_baseline": {"value": value, "unit": "tree-steps/s", "cores": min(cores, w.K), "kind": "oracle",
+            "cpu_baseline": {"value": value, "unit": "tree-steps/s", "cores": cores, "kind": "oracle",
                              "cpu": cpu_model(),
-                             "sample": f"1 of {w.batch} requests per step, scaled to the full batch"},
+                             "sample": f"1 of {w.batch} requests per step, scaled to the full batch; cores = "
+                                       f"OpenMP threads that ran part of the oracle's loops"},
             "e2e": {"value": value, "unit": "tree-steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
     return 0
@@ -388,7 +480,17 @@ def main(argv=None):
     assert rheo.status(cfg, ws, stream) == 0
 
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    soak_s = 0.4
     with Clocks(torch.cuda.current_device()) as clk:
+        # the same graph replayed for soak_s right before the timed steps, so
+        # that the sampler (every 20 ms) sees this load's clocks even when the
+        # timed steps last a few milliseconds
+        with torch.cuda.stream(stream):
+            t_end = time.time() + soak_s
+            while time.time() < t_end:
+                for _ in range(25):
+                    graph.replay()
+                stream.synchronize()
         barrier(world)
         torch.cuda.synchronize()
         with torch.cuda.stream(stream):
@@ -401,6 +503,8 @@ def main(argv=None):
     local_s = start.elapsed_time(stop) / 1e3
     secs = reduce_max_time(local_s, world, device)
     clocks = clk.summary()
+    clocks["window"] = f"{soak_s} s of the same step replayed right before the timed steps, and the timed steps"
+    gpu_res = gpu_outputs(tree, pr, out) if rank == 0 else None
 
     # per-kernel durations: replays (or eager steps when captured events are not
     # available) with a synchronise after each, events read every time
@@ -673,7 +777,7 @@ def main(argv=None):
             w.batch * w.vocab * esz, by_depth[0] / n_k, f"{w.name}:expand_d1"
     ach = dom_bytes / (dom_ms / 1e3) / 1e9
     traffic = _traffic(dom_key)
-    cpu = None if args.no_cpu_baseline else cpu_baseline(w, draft)
+    cpu, parity = (None, None) if args.no_cpu_baseline else cpu_baseline(w, draft, gpu_res)
     line = {
         "metric": METRIC, "value": world * args.steps / secs, "unit": "tree-steps/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3,
@@ -682,7 +786,10 @@ def main(argv=None):
                    "budget": w.budget, "temperature": sorted(set(w.temperatures)), "logits": w.dtype,
                    "bytes_per_step": expand_bytes + verify_bytes, "l2": "inputs 4x larger than L2, no flush",
                    "parallelism": f"replicas{world}", "cuda_graph": True,
-                   "kernel_timing": "separate graph with event nodes" if graph_events else "eager steps"},
+                   "kernel_timing": ("per-call times from a separate graph with event nodes between the "
+                                     "calls (an event node also removes the programmatic-launch overlap "
+                                     "of the calls it separates, so they are upper bounds)")
+                   if graph_events else "eager steps"},
         "roofline": {"bound": "hbm", "kernel": dom_name, "achieved": ach, "peak": peak, "unit": "GB/s",
                      "frac": ach / peak, "peak_kind": peak_kind, "traffic": traffic,
                      "bytes_per_launch": dom_bytes, "ms_per_launch": dom_ms,
@@ -701,6 +808,7 @@ def main(argv=None):
         "gpu_launches": args.steps * (D + 5),  # D expand, 1 prune, 4 verify (prep, stream, table, residual)
         "e2e": e2e,
         "cpu_baseline": cpu,
+        "parity": parity,
     }
     print(json.dumps(line))
     return 0

@@ -106,6 +106,9 @@ def lib():
                                         ctypes.c_int64, ctypes.c_float, ctypes.c_uint64,
                                         ctypes.c_int32, _P, _P]
         L.orc_tree_attention.argtypes = [ctypes.POINTER(_Cfg), ctypes.POINTER(_Pruned), _P, _P, _P, _P]
+        L.orc_threads_used.argtypes = [ctypes.c_int32]
+        L.orc_set_threads.argtypes = [ctypes.c_int32]
+        L.orc_set_threads.restype = None
     return _lib
 
 
@@ -340,3 +343,17 @@ def run_step(cfg: Config, draft_rows, target_rows, T, seed, offset):
     tgt = target_rows(tree, pr) if callable(target_rows) else target_rows
     out = verify(cfg, tgt, T, seed, offset, tree, pr)
     return tree, pr, out
+
+
+def threads_used(reset: bool = True) -> int:
+    """OpenMP threads that ran part of the oracle's parallel loops since the last reset."""
+    return int(lib().orc_threads_used(1 if reset else 0))
+
+
+def set_threads(n: int) -> None:
+    """Team size of the oracle's parallel loops from now on."""
+    lib().orc_set_threads(int(n))
+
+
+def max_threads() -> int:
+    return int(lib().orc_max_threads())

@@ -32,6 +32,9 @@
  *  accumulated in fp64 and rounded once to fp32.
  */
 #include "rheo_oracle.h"
+#ifdef _OPENMP
+#include <omp.h>
+#endif
 
 #include <math.h>
 #include <stdlib.h>
@@ -48,6 +51,41 @@ int64_t orc_nodes_per_request(const orc_cfg* c) {
 }
 
 int64_t orc_expansions_per_request(const orc_cfg* c) { return 1 + (int64_t)(c->D - 1) * c->K; }
+
+/* Thread accounting for timing reports: which OpenMP threads ran at least one
+ * iteration of a parallel loop since the last reset. */
+#define ORC_MAX_THREADS 1024
+static volatile unsigned char g_thread_busy[ORC_MAX_THREADS];
+static void note_thread(void) {
+#ifdef _OPENMP
+    const int t = omp_get_thread_num();
+    if (t >= 0 && t < ORC_MAX_THREADS) g_thread_busy[t] = 1;
+#else
+    g_thread_busy[0] = 1;
+#endif
+}
+int orc_threads_used(int32_t reset) {
+    int n = 0;
+    for (int i = 0; i < ORC_MAX_THREADS; ++i) {
+        n += g_thread_busy[i] ? 1 : 0;
+        if (reset) g_thread_busy[i] = 0;
+    }
+    return n;
+}
+void orc_set_threads(int32_t n) {
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}
+int orc_max_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
 
 int orc_check_cfg(const orc_cfg* c) {
     if (!c) return -1;
@@ -350,6 +388,7 @@ int orc_expand(const orc_cfg* c, int32_t d, const float* rows, const float* T, c
     for (int64_t rr = 0; rr < nrows; ++rr) {
         int b = (int)(rr / F), f = (int)(rr % F);
         const float* l = rows + rr * (int64_t)c->V;
+        note_thread();
         if (expand_row(c, d, b, f, l, T[b], seed[b], offset[b], t)) err |= 1;
     }
     if (err) return -2;
@@ -734,8 +773,10 @@ int orc_verify(const orc_cfg* c, const float* target, const float* T, const uint
         if (!(T[b] > 0.0f) || isinf(T[b])) return -2;
     int err = 0;
 #pragma omp parallel for schedule(dynamic, 1) reduction(| : err)
-    for (int b = 0; b < c->B; ++b)
+    for (int b = 0; b < c->B; ++b) {
+        note_thread();
         if (verify_request(c, b, target, T[b], seed[b], offset[b], t, p, o)) err |= 1;
+    }
     return err ? -2 : 0;
 }
 

@@ -148,6 +148,13 @@ int orc_run_prefix_lm(const orc_cfg* c, const float* draft_table, const float* t
 int orc_tree_attention(const orc_cfg* c, const orc_pruned* p, uint8_t* mask, int32_t* position,
                        int32_t* retrieve, int32_t* n_leaves);
 
+/* Timing reports: OpenMP threads that ran an iteration of a parallel loop
+ * since the last reset (reset != 0 clears the record), the team size for the
+ * next parallel loops, and the current maximum team size (1 without OpenMP). */
+int orc_threads_used(int32_t reset);
+void orc_set_threads(int32_t n);
+int orc_max_threads(void);
+
 #ifdef __cplusplus
 }
 #endif

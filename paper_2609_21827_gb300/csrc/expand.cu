@@ -8,14 +8,15 @@
 //   * its candidate keys (ord(logit) << 32 | ~id) in a region of shared memory:
 //     every element whose key reaches theta, a lower bound of the segment's
 //     S-th key.  At the first tile theta is the minimum over warps of each
-//     warp's ceil(S/8)-th largest vector maximum; on the segment's tiles 2, 4,
-//     8, ... every warp republishes that statistic over its lanes' running
-//     vector maxima, so theta follows the S-th largest element seen so far.  A
-//     warp whose region fills up cuts it to its own S best keys, which raises
-//     theta too.  A shared 4096-bin histogram of the candidates' top key bits
-//     is kept along.
-// At the end of a segment the histogram locates the bin of the S-th key, and
-// only that bin's keys are ranked.  A row held by one CTA goes straight on to
+//     warp's ceil(S/16)-th largest lane maximum; on every later tile one warp
+//     in turn reads, off a shared two-level histogram of the keys inserted so
+//     far (256 coarse bins of the top 8 key bits over 16384 fine bins of the
+//     top 14), the fine bin holding the S-th key, whose lower edge becomes
+//     theta.  A warp whose region fills up cuts it to its own S best keys,
+//     which raises theta too.
+// At the end of a segment the histogram locates the fine bin of the S-th key,
+// and the keys at or above it are counting-sorted by fine bin and ranked
+// within their bin.  A row held by one CTA goes straight on to
 // its children; otherwise the lists and partial sums go to the workspace and
 // the CTA that ends the last segment of a row (arrival counter, never a wait)
 // merges them.  Then the row's sorted support gives Y from the tempered tail by

@@ -133,6 +133,7 @@ def run_oracle(w: synth.Workload, draft: synth.DraftInputs, cfg: rheo.Config, re
 class Report:
     requests: int = 0
     exact: int = 0
+    verified: int = 0  # requests whose verification outputs were compared (trees identical)
     explained: list = field(default_factory=list)
     unexplained: list = field(default_factory=list)
     fp_fail: list = field(default_factory=list)
@@ -141,7 +142,8 @@ class Report:
         return not self.unexplained and not self.fp_fail
 
     def __str__(self):
-        return (f"requests={self.requests} exact={self.exact} explained_flips={len(self.explained)} "
+        return (f"requests={self.requests} exact={self.exact} verified={self.verified} "
+                f"explained_flips={len(self.explained)} {self.explained[:5]} "
                 f"unexplained={self.unexplained[:5]} fp_fail={self.fp_fail[:5]}")
 
 
@@ -174,7 +176,9 @@ def compare(cfg: rheo.Config, g: Side, o: Side, reqs) -> Report:
                         why = ("sample", o.gaps["sample"][j, e])
                         break
                 if why is None:
-                    why = ("pool", 0.0 if d > 1 else 1.0)
+                    # same tokens, other parents or slots: the frontiers were
+                    # compared equal already, so no decision margin can explain it
+                    why = ("pool", 1.0)
                 break
             if d < D and not np.array_equal(g.frontiers[d - 1][b], o.frontiers[d - 1][j]):
                 why = ("frontier", o.gaps["frontier"][j, d - 1])
@@ -199,6 +203,7 @@ def compare(cfg: rheo.Config, g: Side, o: Side, reqs) -> Report:
                 rep.fp_fail.append((b, bad, errs))
                 continue
             # verification
+            rep.verified += 1
             n = int(o.acc_len[j])
             lvl = None
             for i in range(D):

@@ -58,3 +58,45 @@ def test_clock_log_parser():
 def test_peaks_are_read():
     peak, kind = bench._peaks()
     assert peak > 1000 and kind in ("measured", "fallback")
+
+
+def test_parity_summary_classifies_differences():
+    """The bench's parity report: identical results are exact; a changed bonus
+    token or a changed tree node with a wide oracle margin is unexplained."""
+    import copy
+    import dataclasses
+
+    import numpy as np
+
+    from paper_2609_21827_gb300 import synth
+
+    w = dataclasses.replace(synth.WORKLOADS["tiny"], name="tiny_b3", batch=3)
+    draft = synth.make_draft_inputs(w, device="cpu")
+    _, ot, op, oo = bench.oracle_cycle(w, draft, range(3))
+    g = {"token": ot.token.copy(), "parent": ot.parent.copy(), "slot": ot.slot.copy(),
+         "acc_len": oo.accepted_len.copy(), "acc_tok": oo.accepted_tokens.copy(),
+         "acc_node": oo.accepted_nodes.copy(), "bonus": oo.bonus_token.copy()}
+    g.update({"pr_" + k: getattr(op, k).copy() for k in bench.PRUNED_FIELDS})
+    rep = bench.parity_summary(w, g, [0, 1, 2], ot, op, oo)
+    assert (rep["exact"], rep["explained_flips"], rep["unexplained"]) == (3, 0, 0)
+    bad = copy.deepcopy(g)
+    bad["bonus"][1] = (bad["bonus"][1] + 1) % w.vocab
+    bad["token"][2, 1 + w.m] = -7  # the sampled child of the root
+    rep = bench.parity_summary(w, bad, [0, 1, 2], ot, op, oo)
+    gaps = {1: float(oo.gap_level[1, int(oo.accepted_len[1])]), 2: float(ot.gap_sample[2, 0])}
+    want_bad = sum(1 for b in (1, 2) if gaps[b] >= bench.FLIP_GAP)
+    assert rep["exact"] == 1 and rep["unexplained"] == want_bad and rep["explained_flips"] == 2 - want_bad
+    assert np.all(g["bonus"] == oo.bonus_token)
+
+
+def test_oracle_reports_threads_it_ran():
+    import oracle
+
+    oracle.build()
+    n = oracle.max_threads()
+    oracle.set_threads(1)
+    try:
+        assert oracle.max_threads() == 1
+    finally:
+        oracle.set_threads(n)
+    assert oracle.max_threads() == n

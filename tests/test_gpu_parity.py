@@ -145,11 +145,18 @@ def test_replay_is_deterministic_and_offset_moves_draws():
 # the five workloads at full size, oracle on sampled requests
 # --------------------------------------------------------------------------
 
-@pytest.mark.parametrize("name,reqs", [("llama8b", [0]), ("qwen3_batch", [3, 11]), ("serving_mix", [0, 37]),
-                                       ("stress", [101])])
+@pytest.mark.parametrize("name,reqs", [("llama8b", [0]), ("qwen3_batch", list(range(16))),
+                                       ("serving_mix", [0, 9, 18, 27, 37, 45, 54, 63]),
+                                       ("stress", [0, 37, 74, 101, 148, 185, 222, 255])])
 def test_parity_full_size_workloads(name, reqs):
+    """The launch the bench times, compared on sampled requests.  Near-tie
+    flips (oracle margin below 1e-6 at the first divergent decision) are
+    counted and printed; every other request must match through verification,
+    and at most a quarter of the requests may be flips."""
     w = synth.WORKLOADS[name]
-    _run(w, reqs=reqs, max_explained_frac=1.0)
+    _, _, rep = _run(w, reqs=reqs, max_explained_frac=0.25)
+    assert rep.verified + len(rep.explained) >= len(reqs), str(rep)
+    assert rep.verified >= max(1, len(reqs) // 2), str(rep)
 
 
 # --------------------------------------------------------------------------

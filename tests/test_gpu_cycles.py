@@ -33,6 +33,20 @@ def _models(V, k, seed, noise=0.8):
     return draft, target
 
 
+def _law_p(run, tries=2):
+    """p-value of a chi-square law test, taken again on fresh seeds when the
+    first sample falls below 0.01.  Eighteen parametrised law tests at a 1 %
+    level would fail by chance in one run out of six; a wrong law fails every
+    sample of this size (24,000 sequences), a right one fails twice in a row
+    one time in 10^4."""
+    p = 0.0
+    for t in range(tries):
+        p = run(t)
+        if p > 0.01:
+            break
+    return p
+
+
 def _chisq_p(obs, exp):
     keep = exp >= 5
     o = np.append(obs[keep], obs[~keep].sum())
@@ -48,22 +62,26 @@ def test_first_two_tokens_follow_the_target(variant, m, T):
     V, k, B = 16, 1, 6000
     draft, target = _models(V, k, seed=100 + m)
     cfg = rheo.Config(batch=B, vocab=V, K=3, depth=3, budget=8, m=m, support=V, dtype="f32")
-    counts = np.zeros(V * V)
-    for rep in range(2):
-        window = torch.full((B, k), 3, dtype=torch.int64, device="cuda")
-        seed = torch.arange(B, dtype=torch.int64, device="cuda") * 7919 + 1000003 * rep + 17
-        res = cycles.run_cycles(cfg, draft, target, window, torch.full((B,), T), seed, cycles=2, L=2,
-                                variant=variant)
-        st = res.streams.cpu().numpy()
-        assert (st >= 0).all()
-        counts += np.bincount(st[:, 0] * V + st[:, 1], minlength=V * V)
     tab = target.table.cpu().double().numpy() / T
     p1 = np.exp(tab[3] - tab[3].max()); p1 /= p1.sum()
     law = np.zeros(V * V)
     for a in range(V):
         p2 = np.exp(tab[a] - tab[a].max()); p2 /= p2.sum()
         law[a * V:(a + 1) * V] = p1[a] * p2
-    assert _chisq_p(counts, law * counts.sum()) > 0.01
+
+    def run(t):
+        counts = np.zeros(V * V)
+        for rep in range(4 * t, 4 * t + 4):
+            window = torch.full((B, k), 3, dtype=torch.int64, device="cuda")
+            seed = torch.arange(B, dtype=torch.int64, device="cuda") * 7919 + 1000003 * rep + 17
+            res = cycles.run_cycles(cfg, draft, target, window, torch.full((B,), T), seed, cycles=2, L=2,
+                                    variant=variant)
+            st = res.streams.cpu().numpy()
+            assert (st >= 0).all()
+            counts += np.bincount(st[:, 0] * V + st[:, 1], minlength=V * V)
+        return _chisq_p(counts, law * counts.sum())
+
+    assert _law_p(run) > 0.01
 
 
 @pytest.mark.parametrize("variant", [rheo.VERIFY_RHEO, rheo.VERIFY_RRSW, rheo.VERIFY_ONEHOT])
@@ -76,22 +94,26 @@ def test_first_two_tokens_follow_the_target_sparse_support(variant, m, S, T):
     V, k, B = 24, 1, 6000
     draft, target = _models(V, k, seed=300 + m + S)
     cfg = rheo.Config(batch=B, vocab=V, K=3, depth=3, budget=8, m=m, support=S, dtype="f32")
-    counts = np.zeros(V * V)
-    for rep in range(2):
-        window = torch.full((B, k), 5, dtype=torch.int64, device="cuda")
-        seed = torch.arange(B, dtype=torch.int64, device="cuda") * 6007 + 1000033 * rep + 29
-        res = cycles.run_cycles(cfg, draft, target, window, torch.full((B,), T), seed, cycles=2, L=2,
-                                variant=variant)
-        st = res.streams.cpu().numpy()
-        assert (st >= 0).all()
-        counts += np.bincount(st[:, 0] * V + st[:, 1], minlength=V * V)
     tab = target.table.cpu().double().numpy() / T
     p1 = np.exp(tab[5] - tab[5].max()); p1 /= p1.sum()
     law = np.zeros(V * V)
     for a in range(V):
         p2 = np.exp(tab[a] - tab[a].max()); p2 /= p2.sum()
         law[a * V:(a + 1) * V] = p1[a] * p2
-    assert _chisq_p(counts, law * counts.sum()) > 0.01
+
+    def run(t):
+        counts = np.zeros(V * V)
+        for rep in range(4 * t, 4 * t + 4):
+            window = torch.full((B, k), 5, dtype=torch.int64, device="cuda")
+            seed = torch.arange(B, dtype=torch.int64, device="cuda") * 6007 + 1000033 * rep + 29
+            res = cycles.run_cycles(cfg, draft, target, window, torch.full((B,), T), seed, cycles=2, L=2,
+                                    variant=variant)
+            st = res.streams.cpu().numpy()
+            assert (st >= 0).all()
+            counts += np.bincount(st[:, 0] * V + st[:, 1], minlength=V * V)
+        return _chisq_p(counts, law * counts.sum())
+
+    assert _law_p(run) > 0.01
 
 
 def _thm2(p, order, qt, n):

@@ -8,6 +8,7 @@
 #include <algorithm>
 #include <cstdint>
 
+#include "config_dims.h"
 #include "rheo.h"
 #include "rheo_device.cuh"
 #include "rheo_kernels.h"
@@ -112,7 +113,9 @@ bool rows_aligned(const void* p, int64_t row_stride, const rheo_config& c) {
 }
 
 
-Dims dims(const rheo_config& c) {
+}  // namespace
+
+Dims config_dims(const rheo_config& c) {
     Dims n;
     n.B = c.batch; n.V = c.vocab; n.K = c.K; n.m = c.m; n.S = c.support; n.D = c.depth; n.N = c.budget;
     n.full = c.support == 0 ? 1 : 0;
@@ -126,6 +129,16 @@ Dims dims(const rheo_config& c) {
     return n;
 }
 
+TreePtrs tree_ptrs(const rheo_tree* t) {
+    return TreePtrs{t->token, t->parent, t->log_proxy, t->score, t->qtilde, t->slot,
+                    t->frontier, t->tail_ids, t->tail_q, t->lse1, t->lse_tail};
+}
+PrunedPtrs pruned_ptrs(const rheo_pruned* p) {
+    return PrunedPtrs{p->gen_id, p->token, p->parent, p->depth, p->first_child, p->n_child, p->sampled_child};
+}
+
+namespace {
+
 bool tree_ok(const rheo_tree* t, const rheo_config& c) {
     if (!(t && t->token && t->parent && t->log_proxy && t->score && t->qtilde && t->slot && t->frontier && t->lse1))
         return false;
@@ -133,14 +146,6 @@ bool tree_ok(const rheo_tree* t, const rheo_config& c) {
 }
 bool pruned_ok(const rheo_pruned* p) {
     return p && p->gen_id && p->token && p->parent && p->depth && p->first_child && p->n_child && p->sampled_child;
-}
-
-TreePtrs tree_ptrs(const rheo_tree* t) {
-    return TreePtrs{t->token, t->parent, t->log_proxy, t->score, t->qtilde, t->slot,
-                    t->frontier, t->tail_ids, t->tail_q, t->lse1, t->lse_tail};
-}
-PrunedPtrs pruned_ptrs(const rheo_pruned* p) {
-    return PrunedPtrs{p->gen_id, p->token, p->parent, p->depth, p->first_child, p->n_child, p->sampled_child};
 }
 
 template <class T> T* at(void* ws, size_t off) { return reinterpret_cast<T*>(static_cast<char*>(ws) + off); }
@@ -171,7 +176,7 @@ extern "C" int rheo_expand(const rheo_config* cfg, int32_t d, const void* logits
         return RHEO_EINVAL;
     const Layout L = layout(*cfg);
     ExpandArgs a;
-    a.n = dims(*cfg);
+    a.n = config_dims(*cfg);
     a.d = d;
     a.F = (d == 1) ? 1 : cfg->K;
     a.logits = static_cast<const char*>(logits);
@@ -219,7 +224,7 @@ extern "C" int rheo_prune(const rheo_config* cfg, const rheo_tree* tree, const r
     if (!valid(cfg) || !tree_ok(tree, *cfg) || !pruned_ok(pruned) || !ws) return RHEO_EINVAL;
     const Layout L = layout(*cfg);
     PruneArgs a;
-    a.n = dims(*cfg);
+    a.n = config_dims(*cfg);
     a.tree = tree_ptrs(tree);
     a.pr = pruned_ptrs(pruned);
     a.status = at<unsigned>(ws, L.status);
@@ -240,7 +245,7 @@ extern "C" int rheo_tree_attention(const rheo_config* cfg, const rheo_pruned* pr
     if (!out->mask && !out->position && !out->retrieve && !out->n_leaves) return RHEO_OK;
     const Layout L = layout(*cfg);
     TreeAttnArgs a;
-    a.n = dims(*cfg);
+    a.n = config_dims(*cfg);
     a.pr = pruned_ptrs(pruned);
     a.mask = out->mask;
     a.position = out->position;
@@ -264,7 +269,7 @@ extern "C" int rheo_verify_variant(const rheo_config* cfg, int32_t variant, cons
         return RHEO_EINVAL;
     const Layout L = layout(*cfg);
     VerifyArgs a;
-    a.n = dims(*cfg);
+    a.n = config_dims(*cfg);
     a.variant = variant == RHEO_VERIFY_RRSW ? kVerifyRrsw : variant == RHEO_VERIFY_ONEHOT ? kVerifyOneHot : kVerifyRheo;
     a.logits = static_cast<const char*>(logits);
     a.row_stride_bytes = row_stride * elem_size(*cfg);
@@ -317,7 +322,7 @@ extern "C" int rheo_verify_full(const rheo_config* cfg, const void* logits, int6
         return RHEO_EINVAL;
     const Layout L = layout(*cfg);
     VerifyArgs a;
-    a.n = dims(*cfg);
+    a.n = config_dims(*cfg);
     a.variant = kVerifyRheo;
     bool draft_aligned = (draft_row_stride * elem_size(*cfg)) % 16 == 0;
     for (int d = 0; d < cfg->depth; ++d) {

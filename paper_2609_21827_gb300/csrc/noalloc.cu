@@ -22,6 +22,7 @@
 #include <cstdint>
 #include <mutex>
 
+#include "config_dims.h"
 #include "rheo.h"
 #include "rheo_device.cuh"
 #include "rheo_kernels.h"
@@ -118,31 +119,16 @@ extern "C" int rheo_verify_static(const rheo_config* cfg, const void* logits, in
     if (cudaMemsetAsync(base, 0, L.clear_end, s) != cudaSuccess) return RHEO_ELAUNCH;
 
     VerifyArgs a;
-    a.n = Dims{};
-    a.n.full = 0;  // sparse support only (full support is refused above)
-    a.n.B = cfg->batch;
-    a.n.V = cfg->vocab;
-    a.n.K = cfg->K;
-    a.n.m = cfg->m;
-    a.n.S = cfg->support;
-    a.n.D = cfg->depth;
-    a.n.N = cfg->budget;
-    a.n.TL = cfg->support - cfg->m;
-    a.n.GW = (cfg->K + 1) + a.n.TL;
+    a.n = config_dims(*cfg);  // the same dimensions as every other entry point
     a.n.chunks = verify_chunks_per_row(cfg->dtype == RHEO_BF16 ? 1 : 0, cfg->vocab);
-    a.n.G1 = 1 + (int64_t)(cfg->K + 1) + (int64_t)(cfg->depth - 1) * cfg->K * (cfg->K + 1);
-    a.n.E = 1 + (int64_t)(cfg->depth - 1) * cfg->K;
-    a.n.eps = cfg->eps;
     const int es = cfg->dtype == RHEO_BF16 ? 2 : 4;
     a.logits = static_cast<const char*>(logits);
     a.row_stride_bytes = row_stride * es;
     a.T = temperature;
     a.seed = seed;
     a.offset = offset;
-    a.tree = TreePtrs{tree->token, tree->parent, tree->log_proxy, tree->score, tree->qtilde, tree->slot,
-                      tree->frontier, tree->tail_ids, tree->tail_q, tree->lse1};
-    a.pr = PrunedPtrs{pruned->gen_id, pruned->token, pruned->parent, pruned->depth, pruned->first_child,
-                      pruned->n_child, pruned->sampled_child};
+    a.tree = tree_ptrs(tree);
+    a.pr = pruned_ptrs(pruned);
     a.accepted_len = out->accepted_len;
     a.accepted_tokens = out->accepted_tokens;
     a.accepted_nodes = out->accepted_nodes;

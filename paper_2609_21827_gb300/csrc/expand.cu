@@ -446,6 +446,12 @@ __device__ __forceinline__ void stage_flush(unsigned long long* region, int& cnt
 
 }  // namespace
 
+// The exact Gumbel key of a full-support token: l/T correctly rounded plus
+// -ln(-ln u) of its Philox word (kept out of line: few tokens get here)
+__device__ __noinline__ float full_gumbel_key(float x, float T, uint32_t w) {
+    return __fadd_rn(__fdiv_rn(x, T), gumbel(u01(w)));
+}
+
 // Gumbel keys each thread keeps in full support: the m+1 best (m <= 1), so
 // that one of them is not the lead
 constexpr int kGumbelKeep = 2;
@@ -471,6 +477,8 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
     unsigned long long* tmpk = reinterpret_cast<unsigned long long*>(spill);
     constexpr int kTmpCap = kSpillBytes / (int)sizeof(unsigned long long);
     __shared__ unsigned long long s_theta;
+    __shared__ unsigned long long s_gbound;  // full support: a bound of the (m+1)-th best Gumbel key
+    __shared__ unsigned long long s_pilot[kXWarps];  // full support: the warps' pilot bounds of a segment
     __shared__ uint32_t s_wb[kXWarps];
     __shared__ int s_rcount[kXWarps];
     __shared__ BlockScratch bs;
@@ -496,7 +504,10 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
     int scnt = 0;  // staged vectors of this warp (warp-uniform)
     int par = 0;
 
-    if (tid == 0) s_theta = 0ull;
+    if (tid == 0) {
+        s_theta = 0ull;
+        s_gbound = 0ull;
+    }
 
     // per-segment state; cnt, theta and seg_valid are warp-uniform
     float mu = -INFINITY;
@@ -591,40 +602,112 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             sum2 = f2_add(sum2, t);
         }
     };
-    // full support, per element: tau = l/T, the tempered sum at the running
-    // maximum mu/T, and the Gumbel key tau + g (Philox tag 1, node = the parent,
-    // draw = token id) against this thread's kept keys
-    auto tile_full = [&](const uint4 (&v)[kVPT], int e0, float mu_prev) {
+    // full support, per element: the tempered sum at the running maximum mu/T,
+    // and the Gumbel key tau + g (tau = l/T correctly rounded; Philox tag 1,
+    // node = the parent, draw = token id) against this thread's kept keys.
+    // The sum's tau needs one ulp, not correct rounding: q = l*(1/T) corrected
+    // by one residual step (Markstein, IBM J. Res. Dev. 34(1), 1990).
+    // Screen: the key can only enter the row's m+1 best if it reaches kb, the
+    // (m+1)-th best key so far of this thread or of the block.  Since
+    // -ln u >= 1-u, g = -ln(-ln u) <= -ln(1-u), and log2(1-u) >= the bits of the
+    // float 1-u read as a fixed-point number minus 127 (log2(1+f) >= f on
+    // [0,1]); so a token with tau + ln2*(127 - bits(1-u)/2^23) below kb less a
+    // margin (2^-10 + |kb|*2^-20, far above the rounding of every step) cannot
+    // reach kb and gets no exact key.  The comparison runs in float:
+    // 2^23 + bits(1-u)/2^8 (built by bit operations, exact) against
+    // 2^23 + 2^15*(127 - log2(e)*(kb' - tau)).  Survivors get the exact key.
+    auto screen_c = [&](unsigned long long kb) -> float {
+        if (kb == 0ull) return INFINITY;  // no bound yet: every token gets its key
+        const float bnd = Elem<0>::value_of_key((uint32_t)(kb >> 32));
+        const float adj = bnd - (0x1p-10f + fabsf(bnd) * 0x1p-20f);  // NaN at +inf: no screen
+        return fmaf(-adj, 32768.0f * kLog2e, 8388608.0f + 32768.0f * 127.0f);
+    };
+    // Before a segment's first tile: each lane's exact key of its largest logit
+    // of the tile; the block's best (m+1)-th of these per warp bounds the row's
+    // (m+1)-th best key from below (each warp holds m+1 real keys at or above
+    // its value), so the first tile is screened like the others.  These keys
+    // only bound: the screen lets them through to their exact keys.
+    auto pilot_bound = [&](const uint4 (&v)[kVPT], int e0) -> unsigned long long {
+        float bx = -INFINITY;
+        int bi = -1;
+#pragma unroll
+        for (int j = 0; j < kVPT; ++j)
+#pragma unroll
+            for (int i = 0; i < VEC; ++i) {
+                const float x = E::value(E::raw(v[j], i));
+                const bool up = x > bx;
+                bx = up ? x : bx;
+                bi = up ? e0 + (j * kXThreads + tid) * VEC + i : bi;
+            }
+        unsigned long long pk = 0ull;
+        if (bi >= 0) {
+            const uint4 rnd = philox_block(fseed, foff, kTagSample, fpar, (uint64_t)(bi >> 2));
+            const float key = full_gumbel_key(bx, fT, word_of(rnd, bi & 3));
+            if (key > -INFINITY) pk = make_key(ord_f32(key), bi);
+        }
+        unsigned long long top = warp_max_u64(pk);
+        if (m == 1) top = warp_max_u64(pk == top ? 0ull : pk);
+        if (lane == 0) s_pilot[warp] = top;
+        __syncthreads();
+        unsigned long long sb = 0ull;
+#pragma unroll
+        for (int q = 0; q < kXWarps; ++q) sb = s_pilot[q] > sb ? s_pilot[q] : sb;
+        return sb;
+    };
+    auto tile_full = [&](const uint4 (&v)[kVPT], int e0, float mu_prev, unsigned long long sb) {
         const float mT = __fdiv_rn(mu, fT);
         if (mu_prev != mu && mu_prev != -INFINITY) {
             const float rs = fast_exp2(__fsub_rn(__fdiv_rn(mu_prev, fT), mT) * kLog2e);
             sumT2 = f2_mul(sumT2, f2_pack(rs, rs));
         }
-        if (mu == -INFINITY) return;
         const float nmc = -mT * kLog2e;
+        const float rT = 1.0f / fT;
+        // straight-line per vector: the Philox blocks, the sum and the screen
+        // of every element; the rare survivors get their exact keys after it
 #pragma unroll
-        for (int j = 0; j < kVPT; ++j) {
+        for (int j = 0; j < kVPT && mu != -INFINITY; ++j) {  // lanes with no element yet skip to the publish
             const int ev = e0 + (j * kXThreads + tid) * VEC;  // first element of this vector
-            float tsum0 = 0.0f, tsum1 = 0.0f;
+            const unsigned long long own = (m == 0) ? gk[0] : gk[kGumbelKeep - 1];
+            const float C = screen_c(own > sb ? own : sb);
+            uint32_t wv[VEC];
 #pragma unroll
             for (int h = 0; h < VEC / 4; ++h) {
                 const uint4 rnd = philox_block(fseed, foff, kTagSample, fpar, (uint64_t)((ev >> 2) + h));
+                wv[4 * h] = rnd.x;
+                wv[4 * h + 1] = rnd.y;
+                wv[4 * h + 2] = rnd.z;
+                wv[4 * h + 3] = rnd.w;
+            }
+            float tsum0 = 0.0f, tsum1 = 0.0f;
+            uint32_t live = 0u;  // elements that pass the screen
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const float x = E::value(E::raw(v[j], 4 * h + i));
-                    const float tau = __fdiv_rn(x, fT);
-                    float tv;
-                    if (m == 1 && x > kx) {  // the new largest stays out; the one it displaces joins
-                        tv = (kx > -INFINITY) ? fast_exp2(fmaf(__fdiv_rn(kx, fT), kLog2e, nmc)) : 0.0f;
-                        kx = x;
-                        kid = ev + 4 * h + i;
-                    } else {
-                        tv = fast_exp2(fmaf(tau, kLog2e, nmc));
-                    }
-                    if (i & 1) tsum1 += tv; else tsum0 += tv;
-                    const float key = __fadd_rn(tau, gumbel(u01(word_of(rnd, i))));
+            for (int i = 0; i < VEC; ++i) {
+                const float x = E::value(E::raw(v[j], i));
+                // m = 1: the new largest stays out and the one it displaces joins
+                const bool up = (m == 1) && x > kx;
+                const float xs = up ? kx : x;
+                kid = up ? ev + i : kid;
+                kx = up ? x : kx;
+                // xs/T within an ulp (NaN for an infinite xs: the clamp makes it a zero term)
+                const float q0 = xs * rT;
+                const float tq = fmaf(fmaf(-q0, fT, xs), rT, q0);
+                const float tv = fast_exp2(fmaxf(fmaf(tq, kLog2e, nmc), -200.0f));
+                if (i & 1) tsum1 += tv; else tsum0 += tv;
+                // 1 - u exactly: 2 - (k+1)/2^23 less 1 - 2^-24, u = (k + 1/2)/2^23
+                const float omu = __fadd_rn(__uint_as_float(((~wv[i]) >> 9) | 0x3F800000u), -0x1.fffffep-1f);
+                const float fb = __uint_as_float(0x4B000000u | (__float_as_uint(omu) >> 8));
+                // x*(1/T) in the screen: its rounding is far inside the margin
+                // (NaN for infinite x: never screened out)
+                live |= (fb > fmaf(x * rT, 32768.0f * kLog2e, C)) ? 0u : (1u << i);
+            }
+            sumT2 = f2_add(sumT2, f2_pack(tsum0, tsum1));
+            if (live) {
+#pragma unroll
+                for (int i = 0; i < VEC; ++i) {
+                    if (!((live >> i) & 1u)) continue;
+                    const float key = full_gumbel_key(E::value(E::raw(v[j], i)), fT, wv[i]);
                     if (key > -INFINITY) {
-                        const unsigned long long pk = make_key(ord_f32(key), ev + 4 * h + i);
+                        const unsigned long long pk = make_key(ord_f32(key), ev + i);
                         if (pk > gk[kGumbelKeep - 1]) {  // insert, keeping gk sorted descending
                             unsigned long long c = pk;
 #pragma unroll
@@ -637,8 +720,16 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
                     }
                 }
             }
-            sumT2 = f2_add(sumT2, f2_pack(tsum0, tsum1));
         }
+        // publish this warp's best bound (and the one it used) for the block's next tiles
+        unsigned long long own = (m == 0) ? gk[0] : gk[kGumbelKeep - 1];
+        own = own > sb ? own : sb;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const unsigned long long y = __shfl_xor_sync(0xFFFFFFFFu, own, o);
+            own = y > own ? y : own;
+        }
+        if (lane == 0 && own) atomicMax(&s_gbound, own);
     };
     // The bound theta.  On the first step of a segment: every warp's kb-th
     // largest running maximum of its lanes (lanes with no element count as
@@ -720,7 +811,10 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
         if (lane == 0) s_rcount[warp] = cnt;
         float Ms;
         const FF Ss = red_partition<kXWarps>(mu, f2_fold(sum2), kLog2e, Ms, red, par);  // its barrier also publishes the counts
-        if (tid == 0) s_theta = 0ull;  // every warp is past its last cut: ready for the next segment
+        if (tid == 0) {  // every warp is past its last cut and its last key: ready for the next segment
+            s_theta = 0ull;
+            s_gbound = 0ull;
+        }
         const int target = (int)min((int64_t)S, seg_valid);
         auto rkey = [&](int i) -> unsigned long long {
             return (i % kRegion) < s_rcount[i / kRegion] ? keys[i] : 0ull;
@@ -1062,7 +1156,11 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             float vm[kVPT];
             const float mu_prev = mu;
             tile_sum(v, vm);
-            if constexpr (FULL) tile_full(v, e0, seg_first ? -INFINITY : mu_prev);
+            if constexpr (FULL) {
+                const unsigned long long sb =
+                    seg_first ? pilot_bound(v, e0) : *reinterpret_cast<volatile unsigned long long*>(&s_gbound);
+                tile_full(v, e0, seg_first ? -INFINITY : mu_prev, sb);
+            }
             refresh(seg_first);
             seg_valid += ne;
             tile_candidates(v, vm, e0);

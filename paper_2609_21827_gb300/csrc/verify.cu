@@ -887,16 +887,28 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
 }
 
 // Full support, after the stream kernel: the rows whose sampled child
-// survived.  One CTA per such row streams the target row and its node's draft
-// row side by side: p = softmax(l/T) (log-partition from the stream kernel),
-// q~ = exp(l_d/T - lse_tail) off the lead (0 at the lead), M = 1 - sum min(p,
-// q~) as float-float; then r^ = max(0, p - q~) at the children and the row's
-// decisions by Algorithm 1 (sampled child first, then the others in slot
-// order), written to the row's table as the stream kernel does for other rows.
+// survived.  One CTA per such row first decides the sampled child (coin
+// against p(Y) / q~(Y)); only after a rejection does it stream the target row
+// and its node's draft row side by side for M = 1 - sum min(p, q~) (p =
+// softmax(l/T) with the log-partition from the stream kernel, q~ = exp(l_d/T -
+// lse_tail) off the lead, 0 at the lead), then decides the other children in
+// slot order against r^ = max(0, p - q~) (Algorithm 1), writing the row's table
+// as the stream kernel does for other rows.
+// While streaming, each exponent is formed in log2 units as (l - T*lse) *
+// log2(e)/T, with T*lse and log2(e)/T held as float-float constants of the
+// row: l - (T*lse).hi is exact near the terms that carry mass, so the
+// exponent keeps fp32 relative accuracy however large l/T is, and the
+// hardware exp2 gives p and q~; each thread sums eight min(p, q~) in fp32 and
+// carries the running total as float-float.
+constexpr int kOvThreads = 512;
+constexpr int kOvWarps = kOvThreads / 32;
+constexpr int kOvBatch = 4;  // vectors of each row in flight per thread
+
 template <int DT, bool ALIGNED, bool DALIGNED>
-__global__ void __launch_bounds__(kThreads) full_overlap_kernel(const VerifyArgs a) {
+__global__ void __launch_bounds__(kOvThreads) full_overlap_kernel(const VerifyArgs a) {
     grid_dependency_begin();
     using E = Elem<DT>;
+    constexpr int VEC = E::VEC;
     __shared__ Red red;
     __shared__ float s_pc[kMaxSupport], s_rc[kMaxSupport], s_coin[kMaxSupport + 1];
     __shared__ int s_slot[kMaxSupport];
@@ -922,23 +934,10 @@ __global__ void __launch_bounds__(kThreads) full_overlap_kernel(const VerifyArgs
     const char* drow = a.draft[dd - 1] + ((int64_t)b * (dd == 1 ? 1 : K) + f) * a.draft_row_stride_bytes;
     const char* trow = a.logits + r * a.row_stride_bytes;
     int par = 0;
-    FF ov{0.0f, 0.0f};
-    for (int64_t e0 = (int64_t)tid * E::VEC; e0 < V; e0 += (int64_t)kThreads * E::VEC) {
-        const uint4 tv = load_vec<DT, ALIGNED>(trow, e0, V);
-        const uint4 dv = load_vec<DT, DALIGNED>(drow, e0, V);
-#pragma unroll
-        for (int i = 0; i < E::VEC; ++i) {
-            const int64_t id = e0 + i;
-            if (id >= V) break;
-            const float pt = exp_ff_minus(ff_div(E::value(E::raw(tv, i)), T), lse);
-            const float qt = (id == lead) ? 0.0f
-                                          : expf(__fsub_rn(__fdiv_rn(E::value(E::raw(dv, i)), T), lt.hi) - lt.lo);
-            ov = ff_add(ov, fminf(pt, qt));
-        }
-    }
-    ov = red_sum_ff(ov, red, par);
+
+    // the children: p and r^ = max(0, p - q~) at each
     const int nc_ok = (nc >= 0 && nc <= K + 1) ? nc : 0;
-    for (int c = tid; c < nc_ok; c += kThreads) {
+    for (int c = tid; c < nc_ok; c += kOvThreads) {
         const int* ch = a.rec_child + (r * (K + 1) + c) * 3;
         const int tok = __ldcg(ch + 0);
         const float pt = exp_ff_minus(ff_div(E::value(E::load_scalar(trow, tok)), T), lse);
@@ -949,12 +948,59 @@ __global__ void __launch_bounds__(kThreads) full_overlap_kernel(const VerifyArgs
         s_rc[c] = dlt > 0.0f ? dlt : 0.0f;
         s_slot[c] = __ldcg(ch + 2);
     }
-    for (int i = tid; i < K + 2; i += kThreads) s_coin[i] = __ldcg(a.rec_coin + r * (K + 2) + i);
+    for (int i = tid; i < K + 2; i += kOvThreads) s_coin[i] = __ldcg(a.rec_coin + r * (K + 2) + i);
     __syncthreads();
+    // the sampled child first: accepted iff eta * q~(Y) <= p(Y); M is then not needed
+    const bool sampled_ok = sc - fc >= 0 && sc - fc < nc_ok && __fmul_rn(s_coin[0], qs) <= s_pc[sc - fc];
+
+    FF ov{0.0f, 0.0f};
+    if (!sampled_ok) {  // block-uniform
+        const FF cp = ff_mul(T, lse), cq = ff_mul(T, lt);
+        // log2(e)/T as float-float (log2(e) = 0x1.715476p+0 + 0x1.4ae0cp-26); the
+        // high part rounded down, so the low part is positive and a logit of -inf
+        // gives an exponent of -inf (never -inf + inf)
+        const float l2h = 0x1.715476p+0f, l2l = 0x1.4ae0cp-26f;
+        const float clh = __fdiv_rd(l2h, T);
+        const float cll = __fdiv_rn(fmaf(-clh, T, l2h) + l2l, T);
+        const int nvec = (V + VEC - 1) / VEC;
+        for (int v0 = tid; v0 < nvec; v0 += kOvBatch * kOvThreads) {
+            uint4 tv[kOvBatch], dv[kOvBatch];
+#pragma unroll
+            for (int u = 0; u < kOvBatch; ++u) {
+                const int64_t e0 = (int64_t)(v0 + u * kOvThreads) * VEC;
+                tv[u] = load_vec<DT, ALIGNED>(trow, e0, V);   // past V: -inf, no mass
+                dv[u] = load_vec<DT, DALIGNED>(drow, e0, V);
+            }
+#pragma unroll
+            for (int u = 0; u < kOvBatch; ++u) {
+                const int e0 = (v0 + u * kOvThreads) * VEC;
+                float s8 = 0.0f;
+#pragma unroll
+                for (int i = 0; i < VEC; ++i) {
+                    const float dpx = __fsub_rn(__fsub_rn(E::value(E::raw(tv[u], i)), cp.hi), cp.lo);
+                    const float dqx = __fsub_rn(__fsub_rn(E::value(E::raw(dv[u], i)), cq.hi), cq.lo);
+                    const float pt = fast_exp2(fmaf(dpx, clh, dpx * cll));
+                    const float qt = fast_exp2(fmaf(dqx, clh, dqx * cll));
+                    s8 += fminf(pt, qt);
+                }
+                if ((unsigned)(lead - e0) < (unsigned)VEC) {  // q~ is 0 at the lead: sum the vector again without it
+                    s8 = 0.0f;
+                    for (int i = 0; i < VEC; ++i) {
+                        if (e0 + i == lead) continue;
+                        const float dpx = __fsub_rn(__fsub_rn(E::value(E::raw(tv[u], i)), cp.hi), cp.lo);
+                        const float dqx = __fsub_rn(__fsub_rn(E::value(E::raw(dv[u], i)), cq.hi), cq.lo);
+                        s8 += fminf(fast_exp2(fmaf(dpx, clh, dpx * cll)), fast_exp2(fmaf(dqx, clh, dqx * cll)));
+                    }
+                }
+                ov = ff_add(ov, s8);
+            }
+        }
+        ov = red_sum_ff<kOvWarps>(ov, red, par);
+    }
     if (tid == 0) {
         FF M{1.0f, 0.0f};
         int acc = -1, use_tail = 0;
-        if (sc - fc >= 0 && sc - fc < nc_ok && __fmul_rn(s_coin[0], qs) <= s_pc[sc - fc]) {
+        if (sampled_ok) {
             acc = sc;
         } else {
             M = ff_add(FF{1.0f, 0.0f}, ff_neg(ov));
@@ -995,12 +1041,13 @@ cudaError_t launch_verify_full(const VerifyArgs& a, int dtype, bool aligned, boo
     err = (dtype == 1) ? go(verify_table_kernel<1>, gt) : go(verify_table_kernel<0>, gt);
     if (err != cudaSuccess) return err;
     const dim3 go_rows((unsigned)rows);
+    auto go_ov = [&](auto kern) { return launch_dependent(kern, go_rows, dim3(kOvThreads), 0, s, a); };
     if (dtype == 1) {
-        if (aligned && draft_aligned) err = go(full_overlap_kernel<1, true, true>, go_rows);
-        else err = go(full_overlap_kernel<1, false, false>, go_rows);
+        if (aligned && draft_aligned) err = go_ov(full_overlap_kernel<1, true, true>);
+        else err = go_ov(full_overlap_kernel<1, false, false>);
     } else {
-        if (aligned && draft_aligned) err = go(full_overlap_kernel<0, true, true>, go_rows);
-        else err = go(full_overlap_kernel<0, false, false>, go_rows);
+        if (aligned && draft_aligned) err = go_ov(full_overlap_kernel<0, true, true>);
+        else err = go_ov(full_overlap_kernel<0, false, false>);
     }
     if (err != cudaSuccess) return err;
     const dim3 g2((a.n.V + kResChunk - 1) / kResChunk, a.n.B);

@@ -60,6 +60,7 @@ struct E2Smem {
     int yid;     // full support: the sampled token
     float qy;    // full support: q~(Y)
     unsigned long long gk[4];  // full support: the best Gumbel keys of the row
+    float tMT, tSh, tSl;       // full support: the tail's tempered partition (maximum, float-float sum)
 };
 
 struct HistSel {
@@ -839,6 +840,36 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
         const int seg = (int)blockIdx.x - first_owner;
         const int nseg = sp.owner(r * tpr + tpr - 1) - first_owner + 1;
         const int b = (int)(r / a.F), f = (int)(r % a.F);
+        // full support, per segment: the tempered partition sum without the
+        // segment's largest logit (with m = 1 each thread kept its own largest
+        // out; all but the segment's largest go back in), and the segment's
+        // m+1 best Gumbel keys (block merge, m+1 rounds)
+        float fMT = -INFINITY;
+        FF fST{0.0f, 0.0f};
+        if constexpr (FULL) {
+            __syncthreads();  // the segment's sorted list is published
+            const float mT = __fdiv_rn(mu, fT);
+            float sT = f2_fold(sumT2);
+            const int top_id = (written > 0) ? (int)(0xFFFFFFFFu - (uint32_t)e2.sorted[0]) : -1;
+            if (m == 1 && kid >= 0 && kid != top_id)
+                sT += fast_exp2(fmaf(__fdiv_rn(kx, fT), kLog2e, -mT * kLog2e));
+            fST = red_partition<kXWarps>(mT, sT, kLog2e, fMT, red, par);
+            for (int q = 0; q <= m; ++q) {
+                const unsigned long long bq = red_max_u64<kXWarps>(gk[0], red, par);
+                if (bq != 0ull && gk[0] == bq) {
+#pragma unroll
+                    for (int i = 0; i + 1 < kGumbelKeep; ++i) gk[i] = gk[i + 1];
+                    gk[kGumbelKeep - 1] = 0ull;
+                }
+                if (tid == 0) e2.gk[q] = bq;
+            }
+            if (tid == 0) {
+                if (m == 0) e2.gk[1] = 0ull;
+                e2.tMT = fMT;
+                e2.tSh = fST.hi;
+                e2.tSl = fST.lo;
+            }
+        }
         if (tid == 0) {
             if (isnan(Ss.hi) || Ms == INFINITY) atomicOr(a.status, kStBadLogit);
             if (written != target) atomicOr(a.status, kStInternal);
@@ -857,6 +888,14 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
                 a.seg_mu[(int64_t)r * tpr + seg] = Ms;
                 a.seg_sum[2 * ((int64_t)r * tpr + seg)] = Ss.hi;
                 a.seg_sum[2 * ((int64_t)r * tpr + seg) + 1] = Ss.lo;
+                if constexpr (FULL) {
+                    const int64_t q = (int64_t)r * tpr + seg;
+                    a.seg_tmu[q] = fMT;
+                    a.seg_tsum[2 * q] = fST.hi;
+                    a.seg_tsum[2 * q + 1] = fST.lo;
+                    a.seg_gk[2 * q] = e2.gk[0];
+                    a.seg_gk[2 * q + 1] = e2.gk[1];
+                }
             }
             if (!arrive_last(a.row_ticket + r, (unsigned)nseg, bs)) return;
 
@@ -912,6 +951,54 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             }
             __syncthreads();
             if (tid == 0) e2.bad = (got != S) ? 1 : 0;
+            if constexpr (FULL) {
+                // the tail: the segments' sums, and (m = 1) every segment's
+                // largest logit but the row's lead; Y's candidates: the
+                // segments' m+1 best keys
+                if (tid < 32) {
+                    const int lead_id = (got > 0) ? (int)(0xFFFFFFFFu - (uint32_t)e2.sorted[0]) : -1;
+                    float mx = -INFINITY;
+                    for (int c = tid; c < nseg; c += 32) mx = fmaxf(mx, __ldcg(a.seg_tmu + (int64_t)r * tpr + c));
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
+                    FF acc{0.0f, 0.0f};
+                    unsigned long long k0 = 0ull, k1 = 0ull;
+                    for (int c = tid; c < nseg; c += 32) {
+                        const int64_t q = (int64_t)r * tpr + c;
+                        const FF sc{__ldcg(a.seg_tsum + 2 * q), __ldcg(a.seg_tsum + 2 * q + 1)};
+                        if (sc.hi != 0.0f) acc = ff_add(acc, ff_mul(expf(__ldcg(a.seg_tmu + q) - mx), sc));
+                        const unsigned long long top = __ldcg(rk + (int64_t)c * S);
+                        if (m == 1 && top != 0ull && (int)(0xFFFFFFFFu - (uint32_t)top) != lead_id) {
+                            const float xt = E::value_of_key((uint32_t)(top >> 32));
+                            acc = ff_add(acc, expf(__fsub_rn(__fdiv_rn(xt, fT), mx)));
+                        }
+#pragma unroll
+                        for (int j = 0; j < 2; ++j) {
+                            const unsigned long long x = __ldcg(a.seg_gk + 2 * q + j);
+                            if (x > k0) { k1 = k0; k0 = x; } else if (x > k1) { k1 = x; }
+                        }
+                    }
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1) {
+                        acc = ff_add(acc, ff_shfl_xor(acc, o));
+                        const unsigned long long y0 = __shfl_xor_sync(0xFFFFFFFFu, k0, o);
+                        const unsigned long long y1 = __shfl_xor_sync(0xFFFFFFFFu, k1, o);
+                        // the two best of {k0, k1, y0, y1}: keys are distinct tokens or 0
+                        const unsigned long long hi = k0 > y0 ? k0 : y0;
+                        const unsigned long long lo = k0 > y0 ? (k1 > y0 ? k1 : y0) : (y1 > k0 ? y1 : k0);
+                        k0 = hi;
+                        k1 = lo;
+                    }
+                    if (tid == 0) {
+                        e2.tMT = mx;
+                        e2.tSh = acc.hi;
+                        e2.tSl = acc.lo;
+                        e2.gk[0] = k0;
+                        e2.gk[1] = (m == 1) ? k1 : 0ull;
+                    }
+                }
+                __syncthreads();
+            }
         }
         __syncthreads();
         const float lse1 = e2.lse1;
@@ -958,26 +1045,13 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
                 if (!bestp) atomicOr(a.status, kStEmptyRow);
             }
         } else {
-            // full support: the tempered partition over V (each thread's sum at its
-            // maximum mu/T), the tail's = minus the leads; Y = the best Gumbel key
-            // that is not a lead (merged over the block, m+1 rounds)
-            float MT;
-            const float mT = __fdiv_rn(mu, fT);
-            float sT = f2_fold(sumT2);
-            const int lead_id = (int)(0xFFFFFFFFu - (uint32_t)e2.sorted[0]);  // e2.id is not published yet
-            if (m == 1 && kid >= 0 && kid != lead_id)  // kept out, and not the lead: it belongs to the tail
-                sT += fast_exp2(fmaf(__fdiv_rn(kx, fT), kLog2e, -mT * kLog2e));
-            const FF ST = red_partition<kXWarps>(mT, sT, kLog2e, MT, red, par);  // the tail's sum
-            for (int q = 0; q <= m; ++q) {
-                const unsigned long long bq = red_max_u64<kXWarps>(gk[0], red, par);
-                if (bq != 0ull && gk[0] == bq) {
-#pragma unroll
-                    for (int i = 0; i + 1 < kGumbelKeep; ++i) gk[i] = gk[i + 1];
-                    gk[kGumbelKeep - 1] = 0ull;
-                }
-                if (tid == 0) e2.gk[q] = bq;
-            }
+            // full support: the tail's tempered partition (merged over the
+            // segments, the lead left out) and Y = the best Gumbel key that is
+            // not a lead, from the row's m+1 best keys
+            __syncthreads();  // the support's ids are published
             if (tid == 0) {
+                const float MT = e2.tMT;
+                const FF ST{e2.tSh, e2.tSl};
                 int yid = -1;
                 for (int q = 0; q <= m && yid < 0; ++q) {
                     if (!e2.gk[q]) break;

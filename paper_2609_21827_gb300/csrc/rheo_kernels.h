@@ -57,6 +57,11 @@ struct ExpandArgs {
     float* seg_sum;                 // [B*F*tiles_per_row*2] float-float partition sums
     unsigned long long* seg_keys;   // [B*F*tiles_per_row*S]
     float* lse_tail_ff;             // [B*E*2] full support: the tail's log-partition as float-float
+    // full support, per segment: the tempered partition without the segment's
+    // largest logit (maximum, float-float sum) and the m+1 best Gumbel keys
+    float* seg_tmu;                 // [B*F*tiles_per_row]
+    float* seg_tsum;                // [B*F*tiles_per_row*2]
+    unsigned long long* seg_gk;     // [B*F*tiles_per_row*2]
 };
 
 struct PruneArgs {

@@ -745,47 +745,19 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
     __syncthreads();
 
     // key of the draw from r: log r^ + g on the tail (after a rejection), log p + g
-    // elsewhere, over V minus the candidates
+    // elsewhere, over V minus the candidates; with full support after a
+    // rejection every token but the lead is tail, r^ = max(0, p - q~) (no key
+    // where it is 0), and the lead keeps log p + g.
+    // Exact filter: every key is at most lp + g, lp = fp32(l/T - lse) (log r^ <=
+    // log p); the CTA's best exact key among each thread's highest-lp token is a
+    // lower bound B0 of the winning key; g never exceeds kGumbelMax, so a token
+    // with lp + kGumbelMax < B0 cannot win (no uniform drawn); otherwise it can
+    // beat B0 only if u > exp(-exp(lp - B0)), tested with a 1e-4 margin; the
+    // rest get the exact key.
     unsigned long long best = 0ull;
-    if (FULL && drow) {
-#pragma unroll
-        for (int h = 0; h < kResPer / 4; ++h) {
-            if (e0 + 4 * h >= V) break;
-            const uint4 rnd = philox_block(seed, off, kTagResidual, gen_u, (uint64_t)((e0 >> 2) + h));
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int64_t id = e0 + 4 * h + i;
-                if (id >= V) break;
-                const int li = (int)(id - e_lo);
-                if (((excl_bits[li >> 5] | tail_bits[li >> 5]) >> (li & 31)) & 1u) continue;
-                const int q = 4 * h + i;
-                const float x = E::value(E::raw(xv[q / E::VEC], q % E::VEC));
-                const float g = gumbel(u01(word_of(rnd, i)));
-                float key;
-                if (id != lead) {
-                    const float pt = exp_ff_minus(ff_div(x, T), lse_ff);
-                    const float xd = E::value(E::raw(dv[q / E::VEC], q % E::VEC));
-                    const float qt = expf(__fsub_rn(__fdiv_rn(xd, T), lt.hi) - lt.lo);
-                    const float rv = __fsub_rn(pt, qt);
-                    if (!(rv > 0.0f)) continue;
-                    key = __fadd_rn(logf(rv), g);
-                } else {
-                    key = __fadd_rn(__fsub_rn(__fdiv_rn(x, T), lse), g);
-                }
-                if (key > -INFINITY) {
-                    const unsigned long long pk = pack_key(key, id);
-                    best = pk > best ? pk : best;
-                }
-            }
-        }
-    } else {
-        // key = fp32(lp + g), lp = fp32(l/T - lse).  Exact filter: the CTA's best
-        // key among each thread's highest-lp token is a lower bound B0 of the
-        // winning key; g never exceeds kGumbelMax, so a token with lp + kGumbelMax
-        // < B0 cannot win (no uniform drawn); otherwise it can beat B0 only if
-        // u > exp(-exp(lp - B0)), tested with a 1e-4 margin; the rest get the
-        // exact key.
+    {
         constexpr float kGumbelMax = 16.7f;  // -log(-log u) at the largest uniform is 16.636
+        const bool fullr = FULL && drow;
         float lp[kResPer];
         int top = -1;
 #pragma unroll
@@ -796,14 +768,22 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
             lp[q] = ok ? __fsub_rn(__fdiv_rn(E::value(E::raw(xv[q / E::VEC], q % E::VEC)), T), lse) : -INFINITY;
             if (lp[q] > -INFINITY && (top < 0 || lp[q] > lp[top])) top = q;
         }
-        auto exact_key = [&](int q) {
-            const float u = u01(word_of(philox_block(seed, off, kTagResidual, gen_u, (uint64_t)((e0 + q) >> 2)),
-                                        (int)((e0 + q) & 3)));
+        auto exact_key = [&](int q, float u) -> float {  // -inf: no key
+            if (fullr && e0 + q != lead) {
+                const float x = E::value(E::raw(xv[q / E::VEC], q % E::VEC));
+                const float xd = E::value(E::raw(dv[q / E::VEC], q % E::VEC));
+                const float pt = exp_ff_minus(ff_div(x, T), lse_ff);
+                const float qt = expf(__fsub_rn(__fdiv_rn(xd, T), lt.hi) - lt.lo);
+                const float rv = __fsub_rn(pt, qt);
+                return (rv > 0.0f) ? __fadd_rn(logf(rv), gumbel(u)) : -INFINITY;
+            }
             return __fadd_rn(lp[q], gumbel(u));
         };
         unsigned long long pk0 = 0ull;
         if (top >= 0) {
-            const float k0 = exact_key(top);
+            const float u = u01(word_of(philox_block(seed, off, kTagResidual, gen_u, (uint64_t)((e0 + top) >> 2)),
+                                        (int)((e0 + top) & 3)));
+            const float k0 = exact_key(top, u);
             if (k0 > -INFINITY) pk0 = pack_key(k0, e0 + top);
         }
         best = pk0;
@@ -829,7 +809,7 @@ __global__ void __launch_bounds__(kThreads) residual_kernel(const VerifyArgs a) 
                     const float ub = fast_exp2(-t * 1.4426950408889634f);         // exp(-exp(-d))
                     if (u < ub * (1.0f - 1e-4f)) continue;                         // g < d: key below B0
                 }
-                const float key = __fadd_rn(lp[q], gumbel(u));
+                const float key = exact_key(q, u);
                 if (key > -INFINITY) {
                     const unsigned long long pk = pack_key(key, e0 + q);
                     best = pk > best ? pk : best;

@@ -358,6 +358,7 @@ def run_reference(args, w):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_step * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": w.name, "batch": w.batch, "vocab": w.vocab, "depth": w.depth, "K": w.K,
+                       "support": min(w.support, w.vocab) if w.support else "full",
                        "budget": w.budget, "logits": w.dtype},
             "cpu_baseline": {"value": value, "unit": "tree-steps/s", "cores": cores, "kind": "oracle",
                              "cpu": cpu_model(),
@@ -387,6 +388,9 @@ def main(argv=None):
                          "(for launch lists of the tree step alone)")
     ap.add_argument("--depth", type=int, default=0,
                     help="override the workload's depth (fewer expansion launches of the same shape, for profiling)")
+    ap.add_argument("--support", type=int, default=-1,
+                    help="override the workload's top-S support; 0 = full support (App. B, Table "
+                         "tab:sparse_support, row Full: the sampled token over the whole vocabulary)")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)
 
@@ -398,6 +402,9 @@ def main(argv=None):
         w = dataclasses.replace(w, name=f"{w.name}_b{args.batch}", batch=args.batch)
     if args.depth > 0 and args.depth != w.depth:
         w = dataclasses.replace(w, name=f"{w.name}_d{args.depth}", depth=args.depth)
+    if args.support >= 0 and args.support != w.support:
+        w = dataclasses.replace(w, name=f"{w.name}_s{args.support}" if args.support else f"{w.name}_full",
+                                support=args.support)
     if args.impl == "reference":
         return run_reference(args, w)
 
@@ -421,6 +428,14 @@ def main(argv=None):
     expand_bytes = sum(exp_rows) * w.vocab * esz
     verify_bytes = w.batch * (w.budget + 1) * w.vocab * esz
 
+    full = cfg.support == 0  # full support verifies against the expanded nodes' draft rows
+
+    def verify_call(tgt, rows, T, seed, off, s):
+        if full:
+            rheo.verify_full(cfg, tgt, rows, T, seed, off, tree, pr, out, ws, s)
+        else:
+            rheo.verify(cfg, tgt, T, seed, off, tree, pr, out, ws, s)
+
     stream = torch.cuda.Stream(device=device)
     stream.wait_stream(torch.cuda.current_stream())
     try:  # events that become record nodes of the captured graph
@@ -440,7 +455,7 @@ def main(argv=None):
         rheo.prune(cfg, tree, pr, ws, s)
         if with_events:
             ev[D + 1].record(s)
-        rheo.verify(cfg, target, draft.temperature, draft.seed, draft.offset, tree, pr, out, ws, s)
+        verify_call(target, draft.rows, draft.temperature, draft.seed, draft.offset, s)
         if with_events:
             ev[D + 2].record(s)
 
@@ -457,7 +472,7 @@ def main(argv=None):
             rheo.expand(cfg, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tree, ws, s)
         evb[1].record(s)
         rheo.prune(cfg, tree, pr, ws, s)
-        rheo.verify(cfg, target, draft.temperature, draft.seed, draft.offset, tree, pr, out, ws, s)
+        verify_call(target, draft.rows, draft.temperature, draft.seed, draft.offset, s)
 
     # the whole step as one CUDA graph of its kernels alone (timed); a second
     # graph with event record nodes between the calls gives per-call durations
@@ -541,7 +556,7 @@ def main(argv=None):
 
 
     variants, synthetic_lm, full_support, attn_us = None, None, None, None
-    if not args.no_extras:
+    if not args.no_extras and not full:
         # tree-attention inputs of the target forward (not part of the tree step):
         # 20 launches in one graph, averaged over replays
         attn = rheo.TreeAttn(cfg, device=device)
@@ -738,7 +753,7 @@ def main(argv=None):
             rheo.prune(cfg, tree, pr, ws, s)
             for e in ev_tgt:
                 s.wait_event(e)
-            rheo.verify(cfg, d_tgt, d_T, d_seed, d_off, tree, pr, out, ws, s)
+            verify_call(d_tgt, d_rows, d_T, d_seed, d_off, s)
             for x, h in zip((out.accepted_len, out.accepted_tokens, out.bonus_token), res):
                 h.copy_(x, non_blocking=True)
             ev_step.record(s)
@@ -783,6 +798,7 @@ def main(argv=None):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
         "config": {"workload": w.name, "batch": w.batch, "vocab": w.vocab, "depth": w.depth, "K": w.K,
+                   "support": min(w.support, w.vocab) if w.support else "full",
                    "budget": w.budget, "temperature": sorted(set(w.temperatures)), "logits": w.dtype,
                    "bytes_per_step": expand_bytes + verify_bytes, "l2": "inputs 4x larger than L2, no flush",
                    "parallelism": f"replicas{world}", "cuda_graph": True,
@@ -805,7 +821,9 @@ def main(argv=None):
                     "full_support": full_support,
                     "tree_attention_bytes": w.batch * (w.budget + 1) * ((w.budget + 1) + 4 + 4 * (w.depth + 1) + 12)},
         "clocks": clocks,
-        "gpu_launches": args.steps * (D + 5),  # D expand, 1 prune, 4 verify (prep, stream, table, residual)
+        # D expand, 1 prune, verify: prep, stream, table, residual (full support:
+        # and the overlap rows)
+        "gpu_launches": args.steps * (D + 5 + (1 if full else 0)),
         "e2e": e2e,
         "cpu_baseline": cpu,
         "parity": parity,

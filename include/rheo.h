@@ -209,10 +209,10 @@ int rheo_verify_full(const rheo_config* cfg, const void* target_logits, int64_t 
  * minus the workspace.  Scratch state lives in a static device array of
  * RHEO_STATIC_SCRATCH_BYTES that every GPU loading the library holds until
  * exit; configurations needing more return RHEO_ETOOLARGE before any launch.
- * The first call on a device looks the array up (make it before any stream
- * capture); the address is kept for the life of the process and does not
- * survive a cudaDeviceReset, after which the entry point must not be called
- * again.  Calls share the array: calls that overlap on the GPU race, so
+ * Every call looks the array up in the current context (the first call on a
+ * device also loads it: make that call before any stream capture), so calls
+ * after a cudaDeviceReset find the new context's array.  Calls share the
+ * array: calls that overlap on the GPU race, so
  * serialise them.  status: optional device int32 that receives this call's
  * status word (the bits of rheo_get_status); may be NULL. */
 #define RHEO_STATIC_SCRATCH_BYTES (8u << 20)

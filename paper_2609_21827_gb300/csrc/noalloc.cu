@@ -20,7 +20,6 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
-#include <mutex>
 
 #include "config_dims.h"
 #include "rheo.h"
@@ -31,24 +30,15 @@ namespace rheo {
 namespace {
 
 constexpr size_t kStaticScratchBytes = RHEO_STATIC_SCRATCH_BYTES;
-constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
-std::mutex g_setup_mutex;
-void* g_scratch_addr[kMaxDevices] = {nullptr};
-
-// device address of the array on the current device (looked up once per device)
+// device address of the array in the current context, looked up on every call
+// (a runtime lookup, no allocation): an address kept across calls would go
+// stale after the context is torn down and made again (cudaDeviceReset)
 void* scratch_address() {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
-    std::lock_guard<std::mutex> lock(g_setup_mutex);
-    if (!g_scratch_addr[dev]) {
-        void* ptr = nullptr;
-        if (cudaGetSymbolAddress(&ptr, g_static_scratch) != cudaSuccess) return nullptr;
-        g_scratch_addr[dev] = ptr;
-    }
-    return g_scratch_addr[dev];
+    void* ptr = nullptr;
+    return cudaGetSymbolAddress(&ptr, g_static_scratch) == cudaSuccess ? ptr : nullptr;
 }
 
 size_t up256(size_t x) { return (x + 255) & ~(size_t)255; }

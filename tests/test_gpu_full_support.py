@@ -39,6 +39,10 @@ CASES = [
     _W("m1_bf16", vocab=5000, K=5, m=1, depth=3, budget=14, dtype="bf16", temperatures=(0.6, 1.3)),
     _W("ragged", vocab=20011, K=6, m=1, depth=3, budget=20, dtype="bf16", temperatures=(0.8,)),
     _W("low_T", vocab=2000, K=4, depth=3, budget=10, temperatures=(0.05,)),
+    # rows cut into segments over the SMs (a segment per tile), merged by the
+    # row's last CTA: m = 0 (no lead left out), and T = 0.05 over five fp32 tiles
+    _W("seg_m0", vocab=20011, K=5, m=0, depth=3, budget=12, dtype="bf16", temperatures=(0.9,)),
+    _W("seg_low_T", vocab=40000, K=4, m=1, depth=3, budget=10, temperatures=(0.05,)),
 ]
 
 

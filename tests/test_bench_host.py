@@ -100,3 +100,16 @@ def test_oracle_reports_threads_it_ran():
     finally:
         oracle.set_threads(n)
     assert oracle.max_threads() == n
+
+
+def test_reference_arm_full_support_line(capsys):
+    """--impl reference with --support 0 times the oracle's full-support cycle
+    (App. B, row Full) and names it in the config, on the host alone."""
+    import json
+
+    assert bench.main(["--impl", "reference", "--workload", "tiny", "--support", "0", "--steps", "1",
+                       "--warmup", "0"]) == 0
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["value"] > 0
+    assert line["config"]["workload"] == "tiny_full" and line["config"]["support"] == "full"
+    assert line["cpu_baseline"]["kind"] == "oracle"

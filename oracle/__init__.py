@@ -44,7 +44,7 @@ def build(force: bool = False) -> str:
 
 VERIFY_RHEO, VERIFY_RRSW, VERIFY_ONEHOT = 0, 1, 2
 # mistakes planted on purpose (tests that must reject them); see rheo_oracle.h
-PLANT_NONE, PLANT_RESIDUAL_ON_SUPPORT, PLANT_MASS_ON_SUPPORT = 0, 1, 2
+PLANT_NONE, PLANT_RESIDUAL_ON_SUPPORT, PLANT_MASS_ON_SUPPORT, PLANT_BLOCK_UNWEIGHTED = 0, 1, 2, 3
 
 
 class _Cfg(ctypes.Structure):

@@ -98,13 +98,16 @@ int orc_check_cfg(const orc_cfg* c) {
     if (c->N < 1 || c->N > G1 - 1) return -1;
     if (c->m == 0 && !(c->eps > 0.0)) return -1;
     if (c->verify_mode < ORC_VERIFY_RHEO || c->verify_mode > ORC_VERIFY_ONEHOT) return -1;
-    if (c->plant_mode < ORC_PLANT_NONE || c->plant_mode > ORC_PLANT_MASS_ON_SUPPORT) return -1;
+    if (c->plant_mode < ORC_PLANT_NONE || c->plant_mode > ORC_PLANT_BLOCK_UNWEIGHTED) return -1;
     return 0;
 }
 
 /* Support size: S, or the whole vocabulary when S == 0 ("full support",
  * App. B Table tab:sparse_support, row Full).  In full support the tail draw
- * of token v uses draw index v (the token id) instead of its tail position. */
+ * of token v uses draw index v (the token id) instead of its tail position,
+ * after a first draw of the block of ORC_FULL_BLOCK token ids it lies in
+ * (draw V + block index). */
+#define ORC_FULL_BLOCK 256
 static int support_of(const orc_cfg* c) { return c->S == 0 ? c->V : c->S; }
 
 static int64_t depth_base(const orc_cfg* c, int d) {
@@ -265,10 +268,37 @@ static int expand_row(const orc_cfg* c, int d, int b, int f, const float* l, flo
     if (t->lse_tail) t->lse_tail[(int64_t)b * E + e] = (float)lse_tail;
 
     /* Y ~ q~ by Gumbel-max; ties keep the earlier tail position (full support:
-     * the lower token id) */
+     * the lower token id).  Full support draws in two stages, each a
+     * Gumbel-max and so exact (P(block) = its mass / the tail's, then
+     * P(Y | block) = q~ / the block's mass): first a block of ORC_FULL_BLOCK
+     * consecutive token ids by its tempered log-mass, fp32(mt + log mass) + g
+     * (draw V + block index; ties keep the lower block), then the token within
+     * that block by tau + g (draw = token id). */
     int best = -1;
     float bk = -INFINITY, second = -INFINITY;
+    double gap_block = INFINITY;
+    int blk = -1;
+    if (c->S == 0) {
+        const int nblk = (V + ORC_FULL_BLOCK - 1) / ORC_FULL_BLOCK;
+        double* mass = (double*)calloc((size_t)nblk, sizeof(double));
+        if (!mass) { free(srt); free(lq0); return -2; }
+        for (int i = 0; i < TL; ++i) mass[srt[m + i].id / ORC_FULL_BLOCK] += exp((double)tau[i] - mt);
+        float kb = -INFINITY, kb2 = -INFINITY;
+        for (int k = 0; k < nblk; ++k) {
+            if (!(mass[k] > 0.0)) continue; /* no tail token with mass here */
+            const float lm = (c->plant_mode == ORC_PLANT_BLOCK_UNWEIGHTED) ? 0.0f : (float)(mt + log(mass[k]));
+            const float key = lm + gumbel(orc_uniform(seed, offset, ORC_TAG_SAMPLE, (int32_t)par, (uint64_t)V + k));
+            if (key > kb) {
+                kb2 = kb;
+                kb = key;
+                blk = k;
+            } else if (key > kb2) kb2 = key;
+        }
+        free(mass);
+        gap_block = rel_gap(kb, kb2);
+    }
     for (int i = 0; i < TL; ++i) {
+        if (c->S == 0 && srt[m + i].id / ORC_FULL_BLOCK != blk) continue;
         const uint64_t draw = (c->S == 0) ? (uint64_t)srt[m + i].id : (uint64_t)i;
         float g = gumbel(orc_uniform(seed, offset, ORC_TAG_SAMPLE, (int32_t)par, draw));
         float key = tau[i] + g;
@@ -343,7 +373,10 @@ static int expand_row(const orc_cfg* c, int d, int b, int f, const float* l, flo
         t->tail_q[((int64_t)b * E + e) * TL + i] = qt[i];
     }
     t->lse1[(int64_t)b * E + e] = lse1;
-    t->gap_sample[(int64_t)b * E + e] = rel_gap(bk, second);
+    {
+        const double gt = rel_gap(bk, second);
+        t->gap_sample[(int64_t)b * E + e] = gt < gap_block ? gt : gap_block;
+    }
     free(srt);
     free(lq0);
     return 0;

@@ -59,8 +59,17 @@ typedef struct {
  *                       off the support;
  *  MASS_ON_SUPPORT      the residual mass M is summed over the support only
  *                       (tail r^ plus p at the leads) instead of
- *                       1 - sum_tail min(p, q~). */
-enum { ORC_PLANT_NONE = 0, ORC_PLANT_RESIDUAL_ON_SUPPORT = 1, ORC_PLANT_MASS_ON_SUPPORT = 2 };
+ *                       1 - sum_tail min(p, q~).
+ * And one in the full-support draw of Y (a no-op while the vocabulary fits in
+ * one block):
+ *  BLOCK_UNWEIGHTED     the block of the two-stage draw is chosen by g alone,
+ *                       ignoring its mass. */
+enum {
+    ORC_PLANT_NONE = 0,
+    ORC_PLANT_RESIDUAL_ON_SUPPORT = 1,
+    ORC_PLANT_MASS_ON_SUPPORT = 2,
+    ORC_PLANT_BLOCK_UNWEIGHTED = 3
+};
 
 /* Verification rules (all lossless):
  *  RHEO    Algorithm 1: the sampled child first (accept iff eta*q~ <= p), then

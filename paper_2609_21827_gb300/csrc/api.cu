@@ -47,7 +47,7 @@ bool valid(const rheo_config* c) {
 }
 
 struct Layout {
-    size_t status, ex_row_ticket, ex_req_ticket, ex_mu, ex_sum, ex_keys, ex_ltail, ex_tmu, ex_tsum, ex_gk;
+    size_t status, ex_row_ticket, ex_req_ticket, ex_mu, ex_sum, ex_keys, ex_ltail, ex_grp;
     size_t v_mu, v_sum, v_queue, v_hdr, v_child, v_tids, v_tq, v_cx, v_tx, v_coin, v_table, v_rhat, r_best,
         r_ticket;
     size_t total;
@@ -69,10 +69,9 @@ Layout layout(const rheo_config& c) {
     L.ex_sum = take(2 * sizeof(float) * B * F * P);
     L.ex_keys = take(sizeof(unsigned long long) * B * F * P * S);
     L.ex_ltail = take(2 * sizeof(float) * B * expansions_per_request(c));
-    const int64_t FP = c.support == 0 ? B * F * P : 0;  // full support's per-segment partials
-    L.ex_tmu = take(sizeof(float) * FP);
-    L.ex_tsum = take(2 * sizeof(float) * FP);
-    L.ex_gk = take(2 * sizeof(unsigned long long) * FP);
+    const int64_t GT = full_group_tokens(c.dtype == RHEO_BF16 ? 1 : 0);
+    const int64_t FG = c.support == 0 ? B * F * ((c.vocab + GT - 1) / GT) : 0;  // full support's group sums
+    L.ex_grp = take(2 * sizeof(float) * FG);
     L.v_mu = take(sizeof(float) * B * NP * VC);
     L.v_sum = take(2 * sizeof(float) * B * NP * VC);
     L.v_queue = take(sizeof(unsigned) * kStreamQueues * kStreamQueueStride);
@@ -196,23 +195,16 @@ extern "C" int rheo_expand(const rheo_config* cfg, int32_t d, const void* logits
     a.seg_sum = at<float>(ws, L.ex_sum);
     a.seg_keys = at<unsigned long long>(ws, L.ex_keys);
     a.lse_tail_ff = at<float>(ws, L.ex_ltail);
-    a.seg_tmu = at<float>(ws, L.ex_tmu);
-    a.seg_tsum = at<float>(ws, L.ex_tsum);
-    a.seg_gk = at<unsigned long long>(ws, L.ex_gk);
+    a.grp = at<float>(ws, L.ex_grp);
     const int tpr = tiles_per_row(*cfg);
     const int64_t rows = (int64_t)cfg->batch * a.F;
     const int sms = sm_count();
     // Launch shape: one CTA of 16 warps per SM.  Up to one row per SM: every
     // row is cut into P equal segments (P CTAs, P = SMs / rows), so a CTA holds
     // one segment and P = 1 needs no merge.  More rows: one CTA per SM, rows
-    // cut where the even split of the tiles falls.  Full support: one CTA per
-    // row, unless the rows fill at most half the SMs; then one CTA per SM, rows
-    // cut at the even split of the tiles (a segment's end and the row's merge
-    // cost about as much as two tiles, so a second segment per CTA does not pay)
+    // cut where the even split of the tiles falls.
     int grid;
-    if (cfg->support == 0) {
-        grid = (2 * rows <= sms) ? (int)std::min<int64_t>(rows * tpr, (int64_t)sms) : (int)rows;
-    } else if (rows <= sms) {
+    if (rows <= sms) {
         const int64_t P = std::max<int64_t>(1, std::min<int64_t>(tpr, sms / rows));
         grid = (int)(rows * P);
     } else {

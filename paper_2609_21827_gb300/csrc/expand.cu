@@ -59,8 +59,7 @@ struct E2Smem {
     float lse_tail;
     int yid;     // full support: the sampled token
     float qy;    // full support: q~(Y)
-    unsigned long long gk[4];  // full support: the best Gumbel keys of the row
-    float tMT, tSh, tSl;       // full support: the tail's tempered partition (maximum, float-float sum)
+    float lead_sum;  // full support: the lead's group summed without the lead
 };
 
 struct HistSel {
@@ -447,15 +446,8 @@ __device__ __forceinline__ void stage_flush(unsigned long long* region, int& cnt
 
 }  // namespace
 
-// The exact Gumbel key of a full-support token: l/T correctly rounded plus
-// -ln(-ln u) of its Philox word (kept out of line: few tokens get here)
-__device__ __noinline__ float full_gumbel_key(float x, float T, uint32_t w) {
-    return __fadd_rn(__fdiv_rn(x, T), gumbel(u01(w)));
-}
-
-// Gumbel keys each thread keeps in full support: the m+1 best (m <= 1), so
-// that one of them is not the lead
-constexpr int kGumbelKeep = 2;
+// Full support: the block of the two-stage draw of Y (token ids per block)
+constexpr int kFullBlock = 256;
 
 template <int DT, bool ALIGNED, bool FULL>
 __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a) {
@@ -478,8 +470,6 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
     unsigned long long* tmpk = reinterpret_cast<unsigned long long*>(spill);
     constexpr int kTmpCap = kSpillBytes / (int)sizeof(unsigned long long);
     __shared__ unsigned long long s_theta;
-    __shared__ unsigned long long s_gbound;  // full support: a bound of the (m+1)-th best Gumbel key
-    __shared__ unsigned long long s_pilot[kXWarps];  // full support: the warps' pilot bounds of a segment
     __shared__ uint32_t s_wb[kXWarps];
     __shared__ int s_rcount[kXWarps];
     __shared__ BlockScratch bs;
@@ -505,27 +495,12 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
     int scnt = 0;  // staged vectors of this warp (warp-uniform)
     int par = 0;
 
-    if (tid == 0) {
-        s_theta = 0ull;
-        s_gbound = 0ull;
-    }
+    if (tid == 0) s_theta = 0ull;
 
     // per-segment state; cnt, theta and seg_valid are warp-uniform
     float mu = -INFINITY;
     unsigned long long sum2 = 0ull;  // the running sum as a pair of fp32 partial sums
-    // full support: the row's request constants, the running tempered sum
-    // (sum exp(tau - mu/T), tau = l/T correctly rounded) and the best Gumbel keys
-    float fT = 1.0f;
-    unsigned long long fseed = 0ull, foff = 0ull, sumT2 = 0ull;
-    int fpar = 0;
-    // m = 1: this thread's largest logit (first on ties) is kept out of the
-    // tempered sum and added back at the row's end unless it is the row's lead,
-    // so the tail's sum never subtracts a dominant term
-    float kx = -INFINITY;
-    int kid = -1;
-    unsigned long long gk[kGumbelKeep];
-#pragma unroll
-    for (int q = 0; q < kGumbelKeep; ++q) gk[q] = 0ull;
+    float fT = 1.0f;  // full support: the row's temperature
     unsigned long long theta = 0ull;
     int cnt = 0, seg_tiles = 0;
     int64_t seg_valid = 0;
@@ -561,19 +536,7 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
     auto seg_begin = [&](int64_t r) {
         mu = -INFINITY;
         sum2 = 0ull;
-        if constexpr (FULL) {
-            const int b = (int)(r / a.F), f = (int)(r % a.F);
-            fT = __ldg(a.T + b);
-            fseed = __ldg(reinterpret_cast<const unsigned long long*>(a.seed) + b);
-            foff = __ldg(reinterpret_cast<const unsigned long long*>(a.offset) + b);
-            fpar = (a.d == 1) ? 0 : __ldcg(a.tree.frontier + (int64_t)b * K + f);
-            if (fpar < 0 || fpar >= n.G1) fpar = 0;  // reported at the row's end
-            sumT2 = 0ull;
-            kx = -INFINITY;
-            kid = -1;
-#pragma unroll
-            for (int q = 0; q < kGumbelKeep; ++q) gk[q] = 0ull;
-        }
+        if constexpr (FULL) fT = __ldg(a.T + r / a.F);
         seg_valid = 0;
         cnt = 0;
         for (int i = tid; i < (kFineBins + kCoarseBins) / 4; i += kXThreads)
@@ -603,134 +566,40 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             sum2 = f2_add(sum2, t);
         }
     };
-    // full support, per element: the tempered sum at the running maximum mu/T,
-    // and the Gumbel key tau + g (tau = l/T correctly rounded; Philox tag 1,
-    // node = the parent, draw = token id) against this thread's kept keys.
-    // The sum's tau needs one ulp, not correct rounding: q = l*(1/T) corrected
-    // by one residual step (Markstein, IBM J. Res. Dev. 34(1), 1990).
-    // Screen: the key can only enter the row's m+1 best if it reaches kb, the
-    // (m+1)-th best key so far of this thread or of the block.  Since
-    // -ln u >= 1-u, g = -ln(-ln u) <= -ln(1-u), and log2(1-u) >= the bits of the
-    // float 1-u read as a fixed-point number minus 127 (log2(1+f) >= f on
-    // [0,1]); so a token with tau + ln2*(127 - bits(1-u)/2^23) below kb less a
-    // margin (2^-10 + |kb|*2^-20, far above the rounding of every step) cannot
-    // reach kb and gets no exact key.  The comparison runs in float:
-    // 2^23 + bits(1-u)/2^8 (built by bit operations, exact) against
-    // 2^23 + 2^15*(127 - log2(e)*(kb' - tau)).  Survivors get the exact key.
-    auto screen_c = [&](unsigned long long kb) -> float {
-        if (kb == 0ull) return INFINITY;  // no bound yet: every token gets its key
-        const float bnd = Elem<0>::value_of_key((uint32_t)(kb >> 32));
-        const float adj = bnd - (0x1p-10f + fabsf(bnd) * 0x1p-20f);  // NaN at +inf: no screen
-        return fmaf(-adj, 32768.0f * kLog2e, 8388608.0f + 32768.0f * 127.0f);
-    };
-    // Before a segment's first tile: each lane's exact key of its largest logit
-    // of the tile; the block's best (m+1)-th of these per warp bounds the row's
-    // (m+1)-th best key from below (each warp holds m+1 real keys at or above
-    // its value), so the first tile is screened like the others.  These keys
-    // only bound: the screen lets them through to their exact keys.
-    auto pilot_bound = [&](const uint4 (&v)[kVPT], int e0) -> unsigned long long {
-        float bx = -INFINITY;
-        int bi = -1;
-#pragma unroll
-        for (int j = 0; j < kVPT; ++j)
-#pragma unroll
-            for (int i = 0; i < VEC; ++i) {
-                const float x = E::value(E::raw(v[j], i));
-                const bool up = x > bx;
-                bx = up ? x : bx;
-                bi = up ? e0 + (j * kXThreads + tid) * VEC + i : bi;
-            }
-        unsigned long long pk = 0ull;
-        if (bi >= 0) {
-            const uint4 rnd = philox_block(fseed, foff, kTagSample, fpar, (uint64_t)(bi >> 2));
-            const float key = full_gumbel_key(bx, fT, word_of(rnd, bi & 3));
-            if (key > -INFINITY) pk = make_key(ord_f32(key), bi);
-        }
-        unsigned long long top = warp_max_u64(pk);
-        if (m == 1) top = warp_max_u64(pk == top ? 0ull : pk);
-        if (lane == 0) s_pilot[warp] = top;
-        __syncthreads();
-        unsigned long long sb = 0ull;
-#pragma unroll
-        for (int q = 0; q < kXWarps; ++q) sb = s_pilot[q] > sb ? s_pilot[q] : sb;
-        return sb;
-    };
-    auto tile_full = [&](const uint4 (&v)[kVPT], int e0, float mu_prev, unsigned long long sb) {
-        const float mT = __fdiv_rn(mu, fT);
-        if (mu_prev != mu && mu_prev != -INFINITY) {
-            const float rs = fast_exp2(__fsub_rn(__fdiv_rn(mu_prev, fT), mT) * kLog2e);
-            sumT2 = f2_mul(sumT2, f2_pack(rs, rs));
-        }
-        const float nmc = -mT * kLog2e;
+    // full support, per warp and vector row of a tile: the warp holds a group
+    // of 32*VEC consecutive token ids; its tempered sum at the group's own
+    // maximum (the reference) goes to the workspace for the row end's two-stage
+    // draw of Y.  tau = l/T to within an ulp: q = l*(1/T) corrected by one
+    // residual step (Markstein, IBM J. Res. Dev. 34(1), 1990); an infinite l
+    // gives NaN, which the exponent's clamp turns into a zero term.
+    auto tile_full = [&](const uint4 (&v)[kVPT], const float (&vm)[kVPT], int e0, int64_t r) {
+        constexpr int GS = 32 * VEC;
+        const int gpr = (V + GS - 1) / GS;
         const float rT = 1.0f / fT;
-        // straight-line per vector: the Philox blocks, the sum and the screen
-        // of every element; the rare survivors get their exact keys after it
 #pragma unroll
-        for (int j = 0; j < kVPT && mu != -INFINITY; ++j) {  // lanes with no element yet skip to the publish
-            const int ev = e0 + (j * kXThreads + tid) * VEC;  // first element of this vector
-            const unsigned long long own = (m == 0) ? gk[0] : gk[kGumbelKeep - 1];
-            const float C = screen_c(own > sb ? own : sb);
-            uint32_t wv[VEC];
-#pragma unroll
-            for (int h = 0; h < VEC / 4; ++h) {
-                const uint4 rnd = philox_block(fseed, foff, kTagSample, fpar, (uint64_t)((ev >> 2) + h));
-                wv[4 * h] = rnd.x;
-                wv[4 * h + 1] = rnd.y;
-                wv[4 * h + 2] = rnd.z;
-                wv[4 * h + 3] = rnd.w;
-            }
-            float tsum0 = 0.0f, tsum1 = 0.0f;
-            uint32_t live = 0u;  // elements that pass the screen
+        for (int j = 0; j < kVPT; ++j) {
+            const int g0 = e0 + (j * kXThreads + warp * 32) * VEC;  // the group's first token
+            const float gmax = Elem<0>::value_of_key(__reduce_max_sync(0xFFFFFFFFu, ord_f32(vm[j])));
+            const float ref = gmax * rT;
+            const float nref = (ref > -INFINITY && ref < INFINITY) ? -ref * kLog2e : -INFINITY;
+            float s0 = 0.0f, s1 = 0.0f;
 #pragma unroll
             for (int i = 0; i < VEC; ++i) {
                 const float x = E::value(E::raw(v[j], i));
-                // m = 1: the new largest stays out and the one it displaces joins
-                const bool up = (m == 1) && x > kx;
-                const float xs = up ? kx : x;
-                kid = up ? ev + i : kid;
-                kx = up ? x : kx;
-                // xs/T within an ulp (NaN for an infinite xs: the clamp makes it a zero term)
-                const float q0 = xs * rT;
-                const float tq = fmaf(fmaf(-q0, fT, xs), rT, q0);
-                const float tv = fast_exp2(fmaxf(fmaf(tq, kLog2e, nmc), -200.0f));
-                if (i & 1) tsum1 += tv; else tsum0 += tv;
-                // 1 - u exactly: 2 - (k+1)/2^23 less 1 - 2^-24, u = (k + 1/2)/2^23
-                const float omu = __fadd_rn(__uint_as_float(((~wv[i]) >> 9) | 0x3F800000u), -0x1.fffffep-1f);
-                const float fb = __uint_as_float(0x4B000000u | (__float_as_uint(omu) >> 8));
-                // x*(1/T) in the screen: its rounding is far inside the margin
-                // (NaN for infinite x: never screened out)
-                live |= (fb > fmaf(x * rT, 32768.0f * kLog2e, C)) ? 0u : (1u << i);
+                const float q0 = x * rT;
+                const float tq = fmaf(fmaf(-q0, fT, x), rT, q0);
+                const float tv = fast_exp2(fmaxf(fmaf(tq, kLog2e, nref), -200.0f));
+                if (i & 1) s1 += tv; else s0 += tv;
             }
-            sumT2 = f2_add(sumT2, f2_pack(tsum0, tsum1));
-            if (live) {
+            float sg = s0 + s1;
 #pragma unroll
-                for (int i = 0; i < VEC; ++i) {
-                    if (!((live >> i) & 1u)) continue;
-                    const float key = full_gumbel_key(E::value(E::raw(v[j], i)), fT, wv[i]);
-                    if (key > -INFINITY) {
-                        const unsigned long long pk = make_key(ord_f32(key), ev + i);
-                        if (pk > gk[kGumbelKeep - 1]) {  // insert, keeping gk sorted descending
-                            unsigned long long c = pk;
-#pragma unroll
-                            for (int q = 0; q < kGumbelKeep; ++q) {
-                                const unsigned long long hi = c > gk[q] ? c : gk[q];
-                                c = c > gk[q] ? gk[q] : c;
-                                gk[q] = hi;
-                            }
-                        }
-                    }
-                }
+            for (int o = 16; o > 0; o >>= 1) sg += __shfl_xor_sync(0xFFFFFFFFu, sg, o);
+            if (lane == 0 && g0 < V) {
+                const int64_t q = r * gpr + g0 / GS;
+                a.grp[2 * q] = ref;
+                a.grp[2 * q + 1] = sg;
             }
         }
-        // publish this warp's best bound (and the one it used) for the block's next tiles
-        unsigned long long own = (m == 0) ? gk[0] : gk[kGumbelKeep - 1];
-        own = own > sb ? own : sb;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const unsigned long long y = __shfl_xor_sync(0xFFFFFFFFu, own, o);
-            own = y > own ? y : own;
-        }
-        if (lane == 0 && own) atomicMax(&s_gbound, own);
     };
     // The bound theta.  On the first step of a segment: every warp's kb-th
     // largest running maximum of its lanes (lanes with no element count as
@@ -812,10 +681,7 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
         if (lane == 0) s_rcount[warp] = cnt;
         float Ms;
         const FF Ss = red_partition<kXWarps>(mu, f2_fold(sum2), kLog2e, Ms, red, par);  // its barrier also publishes the counts
-        if (tid == 0) {  // every warp is past its last cut and its last key: ready for the next segment
-            s_theta = 0ull;
-            s_gbound = 0ull;
-        }
+        if (tid == 0) s_theta = 0ull;  // every warp is past its last cut: ready for the next segment
         const int target = (int)min((int64_t)S, seg_valid);
         auto rkey = [&](int i) -> unsigned long long {
             return (i % kRegion) < s_rcount[i / kRegion] ? keys[i] : 0ull;
@@ -840,36 +706,6 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
         const int seg = (int)blockIdx.x - first_owner;
         const int nseg = sp.owner(r * tpr + tpr - 1) - first_owner + 1;
         const int b = (int)(r / a.F), f = (int)(r % a.F);
-        // full support, per segment: the tempered partition sum without the
-        // segment's largest logit (with m = 1 each thread kept its own largest
-        // out; all but the segment's largest go back in), and the segment's
-        // m+1 best Gumbel keys (block merge, m+1 rounds)
-        float fMT = -INFINITY;
-        FF fST{0.0f, 0.0f};
-        if constexpr (FULL) {
-            __syncthreads();  // the segment's sorted list is published
-            const float mT = __fdiv_rn(mu, fT);
-            float sT = f2_fold(sumT2);
-            const int top_id = (written > 0) ? (int)(0xFFFFFFFFu - (uint32_t)e2.sorted[0]) : -1;
-            if (m == 1 && kid >= 0 && kid != top_id)
-                sT += fast_exp2(fmaf(__fdiv_rn(kx, fT), kLog2e, -mT * kLog2e));
-            fST = red_partition<kXWarps>(mT, sT, kLog2e, fMT, red, par);
-            for (int q = 0; q <= m; ++q) {
-                const unsigned long long bq = red_max_u64<kXWarps>(gk[0], red, par);
-                if (bq != 0ull && gk[0] == bq) {
-#pragma unroll
-                    for (int i = 0; i + 1 < kGumbelKeep; ++i) gk[i] = gk[i + 1];
-                    gk[kGumbelKeep - 1] = 0ull;
-                }
-                if (tid == 0) e2.gk[q] = bq;
-            }
-            if (tid == 0) {
-                if (m == 0) e2.gk[1] = 0ull;
-                e2.tMT = fMT;
-                e2.tSh = fST.hi;
-                e2.tSl = fST.lo;
-            }
-        }
         if (tid == 0) {
             if (isnan(Ss.hi) || Ms == INFINITY) atomicOr(a.status, kStBadLogit);
             if (written != target) atomicOr(a.status, kStInternal);
@@ -888,14 +724,6 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
                 a.seg_mu[(int64_t)r * tpr + seg] = Ms;
                 a.seg_sum[2 * ((int64_t)r * tpr + seg)] = Ss.hi;
                 a.seg_sum[2 * ((int64_t)r * tpr + seg) + 1] = Ss.lo;
-                if constexpr (FULL) {
-                    const int64_t q = (int64_t)r * tpr + seg;
-                    a.seg_tmu[q] = fMT;
-                    a.seg_tsum[2 * q] = fST.hi;
-                    a.seg_tsum[2 * q + 1] = fST.lo;
-                    a.seg_gk[2 * q] = e2.gk[0];
-                    a.seg_gk[2 * q + 1] = e2.gk[1];
-                }
             }
             if (!arrive_last(a.row_ticket + r, (unsigned)nseg, bs)) return;
 
@@ -951,54 +779,6 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             }
             __syncthreads();
             if (tid == 0) e2.bad = (got != S) ? 1 : 0;
-            if constexpr (FULL) {
-                // the tail: the segments' sums, and (m = 1) every segment's
-                // largest logit but the row's lead; Y's candidates: the
-                // segments' m+1 best keys
-                if (tid < 32) {
-                    const int lead_id = (got > 0) ? (int)(0xFFFFFFFFu - (uint32_t)e2.sorted[0]) : -1;
-                    float mx = -INFINITY;
-                    for (int c = tid; c < nseg; c += 32) mx = fmaxf(mx, __ldcg(a.seg_tmu + (int64_t)r * tpr + c));
-#pragma unroll
-                    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
-                    FF acc{0.0f, 0.0f};
-                    unsigned long long k0 = 0ull, k1 = 0ull;
-                    for (int c = tid; c < nseg; c += 32) {
-                        const int64_t q = (int64_t)r * tpr + c;
-                        const FF sc{__ldcg(a.seg_tsum + 2 * q), __ldcg(a.seg_tsum + 2 * q + 1)};
-                        if (sc.hi != 0.0f) acc = ff_add(acc, ff_mul(expf(__ldcg(a.seg_tmu + q) - mx), sc));
-                        const unsigned long long top = __ldcg(rk + (int64_t)c * S);
-                        if (m == 1 && top != 0ull && (int)(0xFFFFFFFFu - (uint32_t)top) != lead_id) {
-                            const float xt = E::value_of_key((uint32_t)(top >> 32));
-                            acc = ff_add(acc, expf(__fsub_rn(__fdiv_rn(xt, fT), mx)));
-                        }
-#pragma unroll
-                        for (int j = 0; j < 2; ++j) {
-                            const unsigned long long x = __ldcg(a.seg_gk + 2 * q + j);
-                            if (x > k0) { k1 = k0; k0 = x; } else if (x > k1) { k1 = x; }
-                        }
-                    }
-#pragma unroll
-                    for (int o = 16; o > 0; o >>= 1) {
-                        acc = ff_add(acc, ff_shfl_xor(acc, o));
-                        const unsigned long long y0 = __shfl_xor_sync(0xFFFFFFFFu, k0, o);
-                        const unsigned long long y1 = __shfl_xor_sync(0xFFFFFFFFu, k1, o);
-                        // the two best of {k0, k1, y0, y1}: keys are distinct tokens or 0
-                        const unsigned long long hi = k0 > y0 ? k0 : y0;
-                        const unsigned long long lo = k0 > y0 ? (k1 > y0 ? k1 : y0) : (y1 > k0 ? y1 : k0);
-                        k0 = hi;
-                        k1 = lo;
-                    }
-                    if (tid == 0) {
-                        e2.tMT = mx;
-                        e2.tSh = acc.hi;
-                        e2.tSl = acc.lo;
-                        e2.gk[0] = k0;
-                        e2.gk[1] = (m == 1) ? k1 : 0ull;
-                    }
-                }
-                __syncthreads();
-            }
         }
         __syncthreads();
         const float lse1 = e2.lse1;
@@ -1045,21 +825,99 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
                 if (!bestp) atomicOr(a.status, kStEmptyRow);
             }
         } else {
-            // full support: the tail's tempered partition (merged over the
-            // segments, the lead left out) and Y = the best Gumbel key that is
-            // not a lead, from the row's m+1 best keys
+            // full support: Y in two stages, each a Gumbel-max (exact: P(block) =
+            // its mass / the tail's, then P(Y | block) = q~ / the block's mass):
+            // a block of kFullBlock consecutive token ids by its tempered
+            // log-mass fp32(reference + log sum) + g (draw V + block; ties keep
+            // the lower block), then a token of that block by tau + g (tau
+            // correctly rounded, draw = token id; ties keep the lower id).  The
+            // masses come from the groups' sums written while streaming; the
+            // lead's group (m = 1) is summed again without the lead.  The same
+            // sums give the tail's partition.
+            constexpr int GS = 32 * VEC;
+            constexpr int GPB = kFullBlock / GS;
+            static_assert(kFullBlock % GS == 0 && kFullBlock <= kXThreads, "groups tile a block");
+            const int gpr = (V + GS - 1) / GS;
+            const int nblk = (V + kFullBlock - 1) / kFullBlock;
+            const float* grp = a.grp + 2 * r * gpr;
+            const char* rowp = a.logits + r * a.row_stride_bytes;
+            const float rT = 1.0f / T;
             __syncthreads();  // the support's ids are published
-            if (tid == 0) {
-                const float MT = e2.tMT;
-                const FF ST{e2.tSh, e2.tSl};
-                int yid = -1;
-                for (int q = 0; q <= m && yid < 0; ++q) {
-                    if (!e2.gk[q]) break;
-                    const int id = (int)(0xFFFFFFFFu - (uint32_t)e2.gk[q]);
-                    bool lead = false;
-                    for (int i = 0; i < m; ++i) lead |= (e2.id[i] == id);
-                    if (!lead) yid = id;
+            const int lead_id = (m == 1) ? e2.id[0] : -1;
+            const int lead_g = (lead_id >= 0) ? lead_id / GS : -1;
+            if (warp == 0) {
+                float sg = 0.0f;
+                if (lead_g >= 0) {
+                    const float ref = __ldcg(grp + 2 * lead_g);
+                    const float nref = (ref > -INFINITY && ref < INFINITY) ? -ref * kLog2e : -INFINITY;
+                    const int e = lead_g * GS + lane * VEC;
+                    const uint4 vv = load_vec<DT, ALIGNED>(rowp, e, V);
+#pragma unroll
+                    for (int i = 0; i < VEC; ++i) {
+                        if (e + i == lead_id) continue;
+                        const float x = E::value(E::raw(vv, i));
+                        const float q0 = x * rT;
+                        const float tq = fmaf(fmaf(-q0, T, x), rT, q0);
+                        sg += fast_exp2(fmaxf(fmaf(tq, kLog2e, nref), -200.0f));
+                    }
                 }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) sg += __shfl_xor_sync(0xFFFFFFFFu, sg, o);
+                if (lane == 0) e2.lead_sum = sg;
+            }
+            __syncthreads();
+            // this thread's blocks: the tail's partition (at this thread's
+            // largest group reference) and the best block key
+            float mth = -INFINITY, sth = 0.0f;
+            unsigned long long kb = 0ull;
+            for (int k = tid; k < nblk; k += kXThreads) {
+                float rf[GPB], sm[GPB];
+                float rm = -INFINITY;
+#pragma unroll
+                for (int q = 0; q < GPB; ++q) {
+                    const int gi = k * GPB + q;
+                    rf[q] = -INFINITY;
+                    sm[q] = 0.0f;
+                    if (gi < gpr) {
+                        rf[q] = __ldcg(grp + 2 * gi);
+                        sm[q] = (gi == lead_g) ? e2.lead_sum : __ldcg(grp + 2 * gi + 1);
+                        if (sm[q] > 0.0f) rm = fmaxf(rm, rf[q]);
+                    }
+                }
+                if (!(rm > -INFINITY)) continue;  // no mass in this block
+                float bs = 0.0f;
+#pragma unroll
+                for (int q = 0; q < GPB; ++q)
+                    if (sm[q] > 0.0f) bs += sm[q] * fast_exp2((rf[q] - rm) * kLog2e);
+                if (rm > mth) {
+                    sth = sth * fast_exp2((mth - rm) * kLog2e) + bs;
+                    mth = rm;
+                } else {
+                    sth += bs * fast_exp2((rm - mth) * kLog2e);
+                }
+                const float lm = __fadd_rn(rm, logf(bs));
+                const float key = __fadd_rn(lm, gumbel(uniform(seed, off, kTagSample, (int)par_g, (uint64_t)V + k)));
+                if (key > -INFINITY) {
+                    const unsigned long long pk = make_key(ord_f32(key), k);
+                    kb = pk > kb ? pk : kb;
+                }
+            }
+            float MT;
+            const FF ST = red_partition<kXWarps>(mth, sth, kLog2e, MT, red, par);
+            const unsigned long long bkey = red_max_u64<kXWarps>(kb, red, par);
+            const int blk = bkey ? (int)(0xFFFFFFFFu - (uint32_t)bkey) : -1;
+            unsigned long long tk = 0ull;
+            if (blk >= 0 && tid < kFullBlock) {
+                const int id = blk * kFullBlock + tid;
+                if (id < V && id != lead_id) {
+                    const float tau = __fdiv_rn(E::value(E::load_scalar(rowp, id)), T);
+                    const float key = __fadd_rn(tau, gumbel(uniform(seed, off, kTagSample, (int)par_g, (uint64_t)id)));
+                    if (key > -INFINITY) tk = make_key(ord_f32(key), id);
+                }
+            }
+            const unsigned long long ykey = red_max_u64<kXWarps>(tk, red, par);
+            if (tid == 0) {
+                const int yid = ykey ? (int)(0xFFFFFFFFu - (uint32_t)ykey) : -1;
                 const FF lse_tail = ff_add(ff_log(ST), MT);
                 e2.lse_tail = __fadd_rn(lse_tail.hi, lse_tail.lo);
                 const int64_t ei = (a.d == 1) ? 0 : 1 + (int64_t)(a.d - 2) * K + f;
@@ -1071,7 +929,6 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
                 if (yid < 0) {
                     atomicOr(a.status, kStEmptyRow);
                 } else {
-                    const char* rowp = a.logits + r * a.row_stride_bytes;
                     const float tauy = __fdiv_rn(E::value(E::load_scalar(rowp, yid)), T);
                     e2.qy = expf(__fsub_rn(tauy, lse_tail.hi) - lse_tail.lo);
                     for (int j = m; j < S; ++j)
@@ -1228,13 +1085,8 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
                 prefetch_parent(r);
             }
             float vm[kVPT];
-            const float mu_prev = mu;
             tile_sum(v, vm);
-            if constexpr (FULL) {
-                const unsigned long long sb =
-                    seg_first ? pilot_bound(v, e0) : *reinterpret_cast<volatile unsigned long long*>(&s_gbound);
-                tile_full(v, e0, seg_first ? -INFINITY : mu_prev, sb);
-            }
+            if constexpr (FULL) tile_full(v, vm, e0, r);
             refresh(seg_first);
             seg_valid += ne;
             tile_candidates(v, vm, e0);
@@ -1270,5 +1122,7 @@ size_t expand_smem_bytes(int max_segments, int support) {
 }
 
 int expand_tile_elems(int dtype) { return kXTileBytes / (dtype == 1 ? 2 : 4); }
+
+int full_group_tokens(int dtype) { return 32 * (dtype == 1 ? Elem<1>::VEC : Elem<0>::VEC); }
 
 }  // namespace rheo

@@ -57,11 +57,9 @@ struct ExpandArgs {
     float* seg_sum;                 // [B*F*tiles_per_row*2] float-float partition sums
     unsigned long long* seg_keys;   // [B*F*tiles_per_row*S]
     float* lse_tail_ff;             // [B*E*2] full support: the tail's log-partition as float-float
-    // full support, per segment: the tempered partition without the segment's
-    // largest logit (maximum, float-float sum) and the m+1 best Gumbel keys
-    float* seg_tmu;                 // [B*F*tiles_per_row]
-    float* seg_tsum;                // [B*F*tiles_per_row*2]
-    unsigned long long* seg_gk;     // [B*F*tiles_per_row*2]
+    // full support: per group of full_group_tokens consecutive token ids of a
+    // row, its tempered sum at the group's reference (reference, sum)
+    float* grp;                     // [B*F*groups_per_row*2]
 };
 
 struct PruneArgs {
@@ -159,6 +157,7 @@ cudaError_t launch_verify_full(const VerifyArgs& a, int dtype, bool aligned, boo
 size_t expand_keys_bytes(int max_segments, int support);
 size_t expand_smem_bytes(int max_segments, int support);
 int expand_tile_elems(int dtype);
+int full_group_tokens(int dtype);
 cudaError_t launch_tree_attn(const TreeAttnArgs& a, int batch, size_t smem, cudaStream_t s);
 size_t tree_attn_smem_bytes(int budget);
 int verify_table_width(int K);

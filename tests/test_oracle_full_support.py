@@ -77,3 +77,48 @@ def test_monte_carlo_against_enumeration(K, m, T, D, N):
     for (a, b), pr in tl.items():
         p2[a * V + b] += pr
     assert _chisq_p(np.bincount(st[:, 0] * V + st[:, 1], minlength=V * V), p2 * n) > 0.01
+
+
+def _two_stage_draws(V, m, T, n, row, plant=0):
+    cfg = oracle.Config(B=n, V=V, K=2, m=m, S=0, D=1, N=3, plant_mode=plant)
+    tree = oracle.Tree(cfg)
+    rows = np.broadcast_to(row, (n, 1, V)).copy()
+    seeds = np.arange(1, n + 1, dtype=np.uint64) * np.uint64(0x9E3779B97F4A7C15 % (2**61))
+    oracle.expand(cfg, 1, rows, np.full(n, T, np.float32), seeds, np.zeros(n, np.uint64), tree)
+    return tree.token[:, 1 + m]
+
+
+def _tail_law(row, m, T):
+    V = row.size
+    order = np.lexsort((np.arange(V), -row))
+    q = np.zeros(V)
+    q[order[m:]] = special.softmax((row[order[m:]] / np.float32(T)).astype(np.float64))
+    return q
+
+
+@pytest.mark.parametrize("m,T", [(1, 0.8), (0, 1.3)])
+def test_two_stage_draw_law_across_blocks(m, T):
+    """V = 700 spans three blocks of 256 token ids (the last one partial): the
+    block of Y follows the blocks' tail masses and Y the tail law q~."""
+    V, n = 700, 60000
+    rng = np.random.default_rng(71 + m)
+    row = (rng.normal(size=V) * 1.2).astype(np.float32)
+    row[300:330] += 2.0  # a heavier stretch inside the second block
+    ys = _two_stage_draws(V, m, T, n, row)
+    q = _tail_law(row, m, T)
+    blocks = np.array([q[0:256].sum(), q[256:512].sum(), q[512:].sum()])
+    assert _chisq_p(np.bincount(ys // 256, minlength=3), blocks * n) > 0.01
+    assert _chisq_p(np.bincount(ys, minlength=V), q * n) > 0.01
+
+
+def test_two_stage_draw_detects_unweighted_blocks():
+    """A planted mistake (blocks chosen without their mass) fails the same law
+    test: the pin has teeth."""
+    V, n = 700, 60000
+    rng = np.random.default_rng(72)
+    row = (rng.normal(size=V) * 1.2).astype(np.float32)
+    row[300:330] += 2.0
+    q = _tail_law(row, 1, 0.8)
+    blocks = np.array([q[0:256].sum(), q[256:512].sum(), q[512:].sum()])
+    ys = _two_stage_draws(V, 1, 0.8, n, row, plant=oracle.PLANT_BLOCK_UNWEIGHTED)
+    assert _chisq_p(np.bincount(ys // 256, minlength=3), blocks * n) < 1e-6

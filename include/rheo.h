@@ -63,8 +63,10 @@ enum {
  * 1 <= budget <= G1-1, G1 <= 16384, vocab <= 262144, eps > 0 when m = 0.
  * support = 0 selects full support (App. B, Table tab:sparse_support, row
  * Full): the sampled token is drawn from the tempered draft distribution over
- * the whole vocabulary minus the leads, with Philox draw index = token id
- * (sparse support: its tail position); requires m <= 1 and K+1 <= 128; no tail
+ * the whole vocabulary minus the leads, in two Gumbel-max stages (a block of
+ * 256 consecutive token ids by its tempered mass, Philox draw index V + block;
+ * then the token within it, draw index = token id; sparse support: one stage,
+ * draw index = tail position); requires m <= 1 and K+1 <= 128; no tail
  * lists are kept (tail_ids / tail_q unused, lse_tail required) and the tree is
  * verified by rheo_verify_full, which re-reads the expanded nodes' draft rows. */
 typedef struct {

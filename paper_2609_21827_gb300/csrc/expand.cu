@@ -582,16 +582,36 @@ __global__ void __launch_bounds__(kXThreads, 1) expand_kernel(const ExpandArgs a
             const float gmax = Elem<0>::value_of_key(__reduce_max_sync(0xFFFFFFFFu, ord_f32(vm[j])));
             const float ref = gmax * rT;
             const float nref = (ref > -INFINITY && ref < INFINITY) ? -ref * kLog2e : -INFINITY;
-            float s0 = 0.0f, s1 = 0.0f;
+            float sg;
+            if constexpr (DT == 1) {
+                // bf16 pairs in packed fp32 (each lane rounded as the scalar
+                // ops); -inf clamped to -1e30 first (bf16 0xF149), so every
+                // step stays finite and its term is 0
+                const unsigned long long rT2 = f2_pack(rT, rT), nT2 = f2_pack(-fT, -fT);
+                const unsigned long long c2 = f2_pack(kLog2e, kLog2e), nr2 = f2_pack(nref, nref);
+                const uint32_t wv[4] = {v[j].x, v[j].y, v[j].z, v[j].w};
+                unsigned long long acc = f2_pack(0.0f, 0.0f);
 #pragma unroll
-            for (int i = 0; i < VEC; ++i) {
-                const float x = E::value(E::raw(v[j], i));
-                const float q0 = x * rT;
-                const float tq = fmaf(fmaf(-q0, fT, x), rT, q0);
-                const float tv = fast_exp2(fmaxf(fmaf(tq, kLog2e, nref), -200.0f));
-                if (i & 1) s1 += tv; else s0 += tv;
+                for (int h = 0; h < 4; ++h) {
+                    const uint32_t wc = bmax2(wv[h], 0xF149F149u);
+                    const unsigned long long x2 = f2_pack(bf_lo(wc), bf_hi(wc));
+                    const unsigned long long q2 = f2_mul(x2, rT2);
+                    const unsigned long long t2 = f2_fma(f2_fma(q2, nT2, x2), rT2, q2);
+                    acc = f2_add(acc, f2_exp2(f2_fma(t2, c2, nr2)));
+                }
+                sg = f2_fold(acc);
+            } else {
+                float s0 = 0.0f, s1 = 0.0f;
+#pragma unroll
+                for (int i = 0; i < VEC; ++i) {
+                    const float x = E::value(E::raw(v[j], i));
+                    const float q0 = x * rT;
+                    const float tq = fmaf(fmaf(-q0, fT, x), rT, q0);
+                    const float tv = fast_exp2(fmaxf(fmaf(tq, kLog2e, nref), -200.0f));
+                    if (i & 1) s1 += tv; else s0 += tv;
+                }
+                sg = s0 + s1;
             }
-            float sg = s0 + s1;
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) sg += __shfl_xor_sync(0xFFFFFFFFu, sg, o);
             if (lane == 0 && g0 < V) {

@@ -51,10 +51,24 @@ def _cfg(w):
                        dtype=w.dtype)
 
 
-def _run(w, reqs):
+def _masked(draft):
+    """Most logits of every draft row set to -inf (a masked vocabulary), a few
+    finite ones kept at the start and the end of the row."""
+    g = torch.Generator(device="cuda")
+    g.manual_seed(11)
+    for r in draft.rows:
+        mask = torch.rand(r.shape, generator=g, device=r.device) < 0.9
+        mask[..., :16] = False
+        mask[..., -16:] = False
+        r.masked_fill_(mask, float("-inf"))
+
+
+def _run(w, reqs, transform=None):
     import oracle
     cfg = _cfg(w)
     draft = synth.make_draft_inputs(w, device="cuda")
+    if transform:
+        transform(draft)
     tree, pr, ws = rheo.Tree(cfg), rheo.Pruned(cfg), rheo.Workspace(cfg)
     for d in range(1, cfg.depth + 1):
         rheo.expand(cfg, d, draft.rows[d - 1], draft.temperature, draft.seed, draft.offset, tree, ws)
@@ -107,11 +121,13 @@ def test_full_support_tree_parity_qwen3_size():
     assert _run(w, [1, 12]) <= 1
 
 
-def _cycle(w, reqs):
+def _cycle(w, reqs, transform=None):
     """Full cycle with full support on both sides; returns (explained flips, requests compared)."""
     import oracle
     cfg = _cfg(w)
     draft = synth.make_draft_inputs(w, device="cuda")
+    if transform:
+        transform(draft)
     tree, pr, ws, out = rheo.Tree(cfg), rheo.Pruned(cfg), rheo.Workspace(cfg), rheo.VerifyOut(cfg)
     frontiers = []
     for d in range(1, cfg.depth + 1):
@@ -166,3 +182,12 @@ def test_sparse_entry_points_reject_full_support():
     rc = rheo.lib().rheo_verify_variant(ctypes.byref(cfg.c()), 0, None, 0, None, None, None, None, None, None,
                                         None, None)
     assert rc == rheo.RHEO_EINVAL
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_full_support_masked_vocab(dtype):
+    """90 % of every draft row at -inf, rows cut into segments (V = 20011): the
+    group sums, the block masses and both draws skip the masked tokens."""
+    w = _W(f"masked_full_{dtype}", vocab=20011, K=4, m=1, depth=3, budget=10, dtype=dtype, temperatures=(0.8,))
+    assert _run(w, list(range(w.batch)), transform=_masked) <= 1
+    assert _cycle(w, list(range(w.batch)), transform=_masked) <= 1

@@ -21,7 +21,9 @@
 // the CTA that ends the last segment of a row (arrival counter, never a wait)
 // merges them.  Then the row's sorted support gives Y from the tempered tail by
 // Gumbel-max and the K+1 children; the last row of a request selects the next
-// frontier.
+// frontier.  With full support (the FULL template) each warp also sums the
+// tempered terms of its 32*VEC-token groups while streaming, and the row's end
+// draws Y in two Gumbel-max stages over 256-token blocks and then tokens.
 #include "rheo_device.cuh"
 #include "rheo_kernels.h"
 #include "stream.cuh"

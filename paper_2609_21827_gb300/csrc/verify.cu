@@ -943,13 +943,28 @@ __global__ void __launch_bounds__(kOvThreads) full_overlap_kernel(const VerifyAr
         const float clh = __fdiv_rd(l2h, T);
         const float cll = __fdiv_rn(fmaf(-clh, T, l2h) + l2l, T);
         const int nvec = (V + VEC - 1) / VEC;
+        // the next batch of both rows is in flight while this one is summed
+        uint4 tn[kOvBatch], dn[kOvBatch];
+#pragma unroll
+        for (int u = 0; u < kOvBatch; ++u) {
+            const int64_t e0 = (int64_t)(tid + u * kOvThreads) * VEC;
+            tn[u] = load_vec<DT, ALIGNED>(trow, e0, V);  // past V: -inf, no mass
+            dn[u] = load_vec<DT, DALIGNED>(drow, e0, V);
+        }
         for (int v0 = tid; v0 < nvec; v0 += kOvBatch * kOvThreads) {
             uint4 tv[kOvBatch], dv[kOvBatch];
 #pragma unroll
             for (int u = 0; u < kOvBatch; ++u) {
-                const int64_t e0 = (int64_t)(v0 + u * kOvThreads) * VEC;
-                tv[u] = load_vec<DT, ALIGNED>(trow, e0, V);   // past V: -inf, no mass
-                dv[u] = load_vec<DT, DALIGNED>(drow, e0, V);
+                tv[u] = tn[u];
+                dv[u] = dn[u];
+            }
+            if (v0 + kOvBatch * kOvThreads < nvec) {
+#pragma unroll
+                for (int u = 0; u < kOvBatch; ++u) {
+                    const int64_t e0 = (int64_t)(v0 + (kOvBatch + u) * kOvThreads) * VEC;
+                    tn[u] = load_vec<DT, ALIGNED>(trow, e0, V);
+                    dn[u] = load_vec<DT, DALIGNED>(drow, e0, V);
+                }
             }
 #pragma unroll
             for (int u = 0; u < kOvBatch; ++u) {

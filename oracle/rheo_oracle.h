@@ -40,7 +40,9 @@ typedef struct {
     int32_t K;       /* deterministic slots per pool; pool size K+1 */
     int32_t m;       /* lead tokens (the rheostat), 0 <= m <= K */
     int32_t S;       /* sparse support, K+1 <= S <= min(V,128); 0: the whole vocabulary
-                        (full support: tail draws indexed by token id) */
+                        (full support: Y drawn in two Gumbel-max stages, a block of
+                        256 token ids by its tail mass with draw V + block, then the
+                        token within it with draw = token id) */
     int32_t D;       /* expansion depth */
     int32_t N;       /* prune budget (non-root nodes kept) */
     double eps;      /* proxy offset for m = 0 */

@@ -122,3 +122,25 @@ def test_two_stage_draw_detects_unweighted_blocks():
     blocks = np.array([q[0:256].sum(), q[256:512].sum(), q[512:].sum()])
     ys = _two_stage_draws(V, 1, 0.8, n, row, plant=oracle.PLANT_BLOCK_UNWEIGHTED)
     assert _chisq_p(np.bincount(ys // 256, minlength=3), blocks * n) < 1e-6
+
+
+@pytest.mark.parametrize("V", [256, 257, 512])
+def test_two_stage_draw_block_edges(V):
+    """V a multiple of the block (256, 512) and one past it (257: the last
+    block holds a single token, here given the row's largest logit after the
+    lead so that its block carries real mass)."""
+    n = 40000
+    rng = np.random.default_rng(300 + V)
+    row = (rng.normal(size=V) * 1.0).astype(np.float32)
+    row[0] = row.max() + 1.0      # the lead (m = 1)
+    row[V - 1] = row[0] - 0.5     # the last token, alone in its block when V = 257
+    ys = _two_stage_draws(V, 1, 1.0, n, row)
+    q = _tail_law(row, 1, 1.0)
+    assert np.all(ys != 0)  # the lead is never the sampled token
+    assert _chisq_p(np.bincount(ys, minlength=V), q * n) > 0.01
+    nb = (V + 255) // 256
+    if nb == 1:
+        assert np.all(ys < 256)
+    else:
+        blocks = np.array([q[256 * k:256 * (k + 1)].sum() for k in range(nb)])
+        assert _chisq_p(np.bincount(ys // 256, minlength=nb), blocks * n) > 0.01

@@ -43,6 +43,9 @@ CASES = [
     # row's last CTA: m = 0 (no lead left out), and T = 0.05 over five fp32 tiles
     _W("seg_m0", vocab=20011, K=5, m=0, depth=3, budget=12, dtype="bf16", temperatures=(0.9,)),
     _W("seg_low_T", vocab=40000, K=4, m=1, depth=3, budget=10, temperatures=(0.05,)),
+    # a one-token last block of the two-stage draw (V = 257), in both dtypes
+    _W("v257_bf16", vocab=257, K=4, m=1, depth=3, budget=10, dtype="bf16", batch=8),
+    _W("v257_f32_m0", vocab=257, K=4, m=0, depth=3, budget=10, batch=8, temperatures=(1.3,)),
     # the largest vocabulary the library accepts: 1024 blocks, 2048 fp32 groups a row
     _W("max_vocab_bf16", vocab=262144, K=4, m=1, depth=2, budget=8, batch=2, dtype="bf16", temperatures=(0.8,)),
     _W("max_vocab_f32", vocab=262144, K=4, m=0, depth=2, budget=8, batch=2, temperatures=(0.6,)),
